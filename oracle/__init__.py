@@ -1,0 +1,199 @@
+"""Plain fp64 CPU oracle for the DREAM-S tree verification step.
+
+TEST INFRASTRUCTURE. Only the test suite, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import this package. The CUDA library in
+``paper_2606_00535_gb300`` never imports it, and this package imports nothing
+from there: the two share no code.
+
+The arithmetic lives in ``oracle.c`` (straight double-precision loops, one
+thread); this module only marshals numpy arrays into it. Each wrapper names the
+paper passage its C routine follows:
+
+* :func:`tree_attention` -- softmax(scale * q K^T) V of each draft-tree query
+  over the prefix cache plus its own ancestors (paper Sec. 2 "Speculative
+  decoding": one parallel target pass over the drafts; Sec. 2 "Vision-Language
+  Models": cached visual and text tokens take part in every decoding step;
+  Sec. 3.2: attention = softmax(Q K^T / sqrt(z))).
+* :func:`argmax` -- the target's greedy (temperature 0) prediction per node
+  (Sec. 2 "Speculative decoding"; Table 2, Temperature = 0).
+* :func:`accept_path` -- sequential acceptance with the target's token
+  replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
+* :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
+  (Sec. 2 "Vision-Language Models": the cache persists across steps).
+* :func:`ancestor_mask` -- the tree mask the attention uses, for inspection.
+
+Parity of this oracle against the paper's own numbers is unpinned for every
+routine: the paper prints no worked example of this step. Each routine is
+pinned instead by closed forms, special cases that reduce to library
+routines, brute force on tiny inputs and invariants (see ``tests/``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+BAD_PARENT = 0x1
+BAD_TREE_LEN = 0x2
+BAD_KV_LEN = 0x4
+BAD_PAGE = 0x8
+
+
+def build(force: bool = False) -> str:
+    """Compile ``oracle.c`` into ``liboracle.so`` with gcc (no fast-math)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(
+            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math",
+             "-ffp-contract=off", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def _load() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        _lib = ctypes.CDLL(build())
+        i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+        p = ctypes.c_void_p
+        _lib.oracle_ancestor_mask.argtypes = [p, i32, p]
+        _lib.oracle_ancestor_mask.restype = ctypes.c_int
+        _lib.oracle_tree_attention.argtypes = [
+            p, p, p, i64, p, i64, i64, i64, p, p, p, i64, i64, i64, i64, i64, f64, p, i64, p, p]
+        _lib.oracle_tree_attention.restype = ctypes.c_int
+        _lib.oracle_argmax_f32.argtypes = [p, i64, i64, i64, p]
+        _lib.oracle_argmax_f32.restype = None
+        _lib.oracle_argmax_bf16.argtypes = [p, i64, i64, i64, p]
+        _lib.oracle_argmax_bf16.restype = None
+        _lib.oracle_accept_path.argtypes = [p, p, p, p, p, i64, i64, i64, p, p, p, p]
+        _lib.oracle_accept_path.restype = ctypes.c_int
+        _lib.oracle_kv_compact.argtypes = [
+            p, p, i64, i64, i64, p, i64, i64, i64, i64, i64, i64, p, p, p, i64]
+        _lib.oracle_kv_compact.restype = ctypes.c_int
+    return _lib
+
+
+def _ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+
+
+def ancestor_mask(parent) -> np.ndarray:
+    """[T, T] uint8: mask[i, a] = 1 iff a is i or an ancestor of i."""
+    par = _c(parent, np.int32)
+    T = par.shape[0]
+    out = np.zeros((T, T), dtype=np.uint8)
+    st = _load().oracle_ancestor_mask(_ptr(par), T, _ptr(out))
+    if st:
+        raise ValueError(f"malformed tree (status {st:#x})")
+    return out
+
+
+class KVLayout:
+    """How one layer's K/V cache is laid out (see ``oracle.c``).
+
+    ``page_table is None``: contiguous ``[B, capacity, Hkv, D]``.
+    Otherwise paged ``[num_pages, page_size, Hkv, D]`` with
+    ``page_table[B, pages_per_seq]`` physical page ids.
+    """
+
+    def __init__(self, capacity, Hkv, D, page_table=None, page_size=64, num_pages=0):
+        self.capacity = int(capacity)
+        self.Hkv = int(Hkv)
+        self.D = int(D)
+        self.page_table = None if page_table is None else _c(page_table, np.int32)
+        self.page_size = int(page_size)
+        self.pages_per_seq = 0 if page_table is None else int(self.page_table.shape[1])
+        self.num_pages = int(num_pages)
+
+
+def tree_attention(q_bits, k_bits, v_bits, layout: KVLayout, parent, tree_len, kv_len,
+                   Hq: int, scale: float, sel=None):
+    """fp64 tree-masked attention for the selected (b, t, h) triples.
+
+    q_bits: uint16 bf16 patterns [B, T_max, Hq, D]; k_bits / v_bits: uint16
+    patterns of one layer cache. ``sel`` is an [n, 3] int array of (b, t, h);
+    None selects every valid row (t < tree_len[b]). Returns (out [n, D],
+    lse [n], sel, status).
+    """
+    q = _c(q_bits, np.uint16)
+    k = _c(k_bits, np.uint16)
+    v = _c(v_bits, np.uint16)
+    par = _c(parent, np.int32)
+    tl = _c(tree_len, np.int32)
+    kl = _c(kv_len, np.int32)
+    B, T_max, _, D = q.shape
+    if sel is None:
+        sel = np.array([(b, t, h) for b in range(B) for t in range(int(tl[b]))
+                        for h in range(Hq)], dtype=np.int32).reshape(-1, 3)
+    sel = _c(sel, np.int32).reshape(-1, 3)
+    n = sel.shape[0]
+    out = np.empty((n, D), dtype=np.float64)
+    lse = np.empty((n,), dtype=np.float64)
+    st = _load().oracle_tree_attention(
+        _ptr(q), _ptr(k), _ptr(v), layout.capacity, _ptr(layout.page_table), layout.page_size,
+        layout.pages_per_seq, layout.num_pages, _ptr(par), _ptr(tl), _ptr(kl), B, T_max, Hq,
+        layout.Hkv, D, float(scale), _ptr(sel), n, _ptr(out), _ptr(lse))
+    return out, lse, sel, st
+
+
+def argmax(logits, V: Optional[int] = None, bf16_bits: bool = False) -> np.ndarray:
+    """Row-wise argmax of a 2-D array (float32, or uint16 bf16 patterns)."""
+    x = np.asarray(logits)
+    rows = x.shape[0]
+    V = x.shape[1] if V is None else int(V)
+    out = np.empty((rows,), dtype=np.int32)
+    if bf16_bits:
+        x = _c(x, np.uint16)
+        _load().oracle_argmax_bf16(_ptr(x), rows, V, x.shape[1], _ptr(out))
+    else:
+        x = _c(x, np.float32)
+        _load().oracle_argmax_f32(_ptr(x), rows, V, x.shape[1], _ptr(out))
+    return out
+
+
+def accept_path(am, parent, tokens, tree_len, kv_len, max_path: int):
+    """Greedy tree acceptance. Returns dict of accept_len, path, out_tokens,
+    new_kv_len and the OR of data-error bits."""
+    am = _c(am, np.int32)
+    par = _c(parent, np.int32)
+    tok = _c(tokens, np.int32)
+    tl = _c(tree_len, np.int32)
+    kl = _c(kv_len, np.int32)
+    B, T_max = par.shape
+    acc = np.empty((B,), np.int32)
+    path = np.empty((B, max_path), np.int32)
+    outt = np.empty((B, max_path), np.int32)
+    nkl = np.empty((B,), np.int32)
+    st = _load().oracle_accept_path(_ptr(am), _ptr(par), _ptr(tok), _ptr(tl), _ptr(kl), B, T_max,
+                                    max_path, _ptr(acc), _ptr(path), _ptr(outt), _ptr(nkl))
+    return {"accept_len": acc, "path": path, "out_tokens": outt, "new_kv_len": nkl, "status": st}
+
+
+def kv_compact(k_bits, v_bits, layout: KVLayout, kv_len, accept_len, path, n_layers: int = 1,
+               layer_stride: int = 0):
+    """In-place compaction on copies of the caches. Returns (k, v, status)."""
+    k = np.array(k_bits, dtype=np.uint16, copy=True, order="C")
+    v = np.array(v_bits, dtype=np.uint16, copy=True, order="C")
+    kl = _c(kv_len, np.int32)
+    acc = _c(accept_len, np.int32)
+    pth = _c(path, np.int32)
+    B, max_path = pth.shape
+    st = _load().oracle_kv_compact(
+        _ptr(k), _ptr(v), n_layers, layer_stride, layout.capacity, _ptr(layout.page_table),
+        layout.page_size, layout.pages_per_seq, layout.num_pages, layout.Hkv, layout.D, B,
+        _ptr(kl), _ptr(acc), _ptr(pth), max_path)
+    return k, v, st
