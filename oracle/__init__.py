@@ -44,6 +44,7 @@ BAD_PARENT = 0x1
 BAD_TREE_LEN = 0x2
 BAD_KV_LEN = 0x4
 BAD_PAGE = 0x8
+BAD_PATH = 0x10
 
 
 def build(force: bool = False) -> str:

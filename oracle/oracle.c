@@ -63,6 +63,7 @@
 #define ORACLE_BAD_TREE_LEN 0x2
 #define ORACLE_BAD_KV_LEN 0x4
 #define ORACLE_BAD_PAGE 0x8
+#define ORACLE_BAD_PATH 0x10
 
 static double bf16_bits_to_double(uint16_t h) {
   uint32_t u = ((uint32_t)h) << 16;
@@ -356,8 +357,10 @@ int oracle_accept_path(const int32_t *am, const int32_t *parent, const int32_t *
  *     tmp[x] = cache[b, L_b + path[b][x]]   for x = 0 .. A-1   (all reads)
  *     cache[b, L_b + x] = tmp[x]            for x = 0 .. A-1   (then writes)
  * Every other slot keeps its bytes. k, v: bf16 bits, n_layers caches each
- * layer_stride elements apart. Returns data-error bits (bad page ids, path
- * entries outside [0, capacity - L_b)); such a sequence is left untouched.
+ * layer_stride elements apart. A path is what the acceptance walk returns:
+ * path[0] = 0 and strictly increasing. Returns data-error bits (a path that
+ * is not of that form, slots beyond the capacity, bad page ids); such a
+ * sequence is left untouched.
  */
 int oracle_kv_compact(uint16_t *k, uint16_t *v, int64_t n_layers, int64_t layer_stride,
                       int64_t capacity, const int32_t *page_table, int64_t page_size,
@@ -372,9 +375,12 @@ int oracle_kv_compact(uint16_t *k, uint16_t *v, int64_t n_layers, int64_t layer_
     if (A <= 0) continue;
     int bad = 0;
     if (A > max_path || L < 0) bad = ORACLE_BAD_KV_LEN;
+    if (!bad && path[b * max_path] != 0) bad = ORACLE_BAD_PATH;
+    for (int64_t x = 1; !bad && x < A; ++x)
+      if (path[b * max_path + x] <= path[b * max_path + x - 1]) bad = ORACLE_BAD_PATH;
     for (int64_t x = 0; !bad && x < A; ++x) {
       int64_t src = path[b * max_path + x];
-      if (src < 0 || L + src >= capacity || L + x >= capacity) bad = ORACLE_BAD_KV_LEN;
+      if (L + src >= capacity || L + x >= capacity) bad = ORACLE_BAD_KV_LEN;
       else if (kv_row_offset(&lay, b, L + src, 0) < 0 || kv_row_offset(&lay, b, L + x, 0) < 0)
         bad = ORACLE_BAD_PAGE;
     }

@@ -274,3 +274,8 @@ def test_compaction_bad_path_untouched():
     assert st & oracle.BAD_KV_LEN
     np.testing.assert_array_equal(ko[0], k[0])
     np.testing.assert_array_equal(ko[1, 4], k[1, 4])
+    for bad_path in ([1, 2, -1], [0, 2, 2], [0, 3, 1]):
+        ko, _, st = oracle.kv_compact(k, k, lay, np.array([2, 2]), np.array([3, 0]),
+                                      np.array([bad_path, [0, 1, 2]], np.int32))
+        assert st == oracle.BAD_PATH
+        np.testing.assert_array_equal(ko, k)
