@@ -1,0 +1,399 @@
+#!/usr/bin/env python
+"""Verification-step benchmark on one GB300 (replicas on N GPUs under torchrun).
+
+One step = the whole hot path over one batch of draft trees:
+  1. dreams_tree_verify_attn  (tree-masked attention, one layer)
+  2. dreams_verify_step       (argmax of every tree node's logits row, greedy
+                               acceptance walk, KV compaction of the accepted
+                               nodes)
+on device-resident synthetic inputs shaped like the chosen workload
+(default: the batched-serving workload, the largest one). Timing: CUDA events
+on the launching stream around exactly --steps steps after --warmup untimed
+steps, bracketed by barrier + synchronize; inputs rotate over two copies so a
+step never finds its inputs in L2 from the previous step (each copy is larger
+than L2). Prints one JSON line.
+
+--impl reference times the CPU oracle (plain fp64 C, one thread) on a bounded
+sample of the same workload per step and scales it to a full step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import workloads as W  # noqa: E402
+
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="dreams", choices=["dreams", "reference"])
+    ap.add_argument("--config", default="batched", choices=[s.name for s in W.SPECS])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- accounting
+def attn_bytes(w: W.Workload) -> int:
+    """Algorithmic bytes of one attention launch: every K and V row read once
+    (prefix + tree slots, per KV head), Q read and O written once (tree rows)."""
+    kv_tokens = int((w.kv_len + w.tree_len).sum())
+    q_rows = int(w.tree_len.sum())
+    return kv_tokens * w.Hkv * w.D * 2 * 2 + 2 * q_rows * w.Hq * w.D * 2
+
+
+def argmax_bytes(w: W.Workload) -> int:
+    """Algorithmic bytes of the argmax: every logit of every tree node once."""
+    return int(w.tree_len.sum()) * w.V * (4 if w.logits_dtype == "f32" else 2)
+
+
+def attn_flops(w: W.Workload) -> int:
+    return int(sum(4 * int(w.tree_len[b]) * w.Hq * (int(w.kv_len[b]) + int(w.tree_len[b])) * w.D
+                   for b in range(w.B)))
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- dreams arm
+def run_dreams(args, rank, world, local):
+    import paper_2606_00535_gb300 as dreams
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = W.make(args.config, seed=None if rank == 0 else 20260 + 97 * rank + W.SPEC_BY_NAME[args.config].index)
+    max_path = w.max_path
+    copies = []
+    for _ in range(2):
+        c = {
+            "q": w.q.to(dev), "k": w.k.to(dev), "v": w.v.to(dev),
+            "pt": None if w.page_table is None else w.page_table.to(dev),
+            "parent": w.parent.to(dev), "tokens": w.tokens.to(dev), "tree_len": w.tree_len.to(dev),
+            "kv_len": w.kv_len.to(dev), "logits": w.logits.to(dev),
+        }
+        c["kv"] = dreams.KVCache(c["k"], c["v"], c["pt"])
+        c["tree"] = dreams.Tree(c["parent"], c["tokens"], c["tree_len"], c["kv_len"])
+        c["out"] = torch.empty_like(c["q"])
+        c["outs"] = (torch.empty(w.B, dtype=torch.int32, device=dev),
+                     torch.empty((w.B, max_path), dtype=torch.int32, device=dev),
+                     torch.empty((w.B, max_path), dtype=torch.int32, device=dev),
+                     torch.empty(w.B, dtype=torch.int32, device=dev))
+        copies.append(c)
+    copy_bytes = sum(t.numel() * t.element_size() for t in (copies[0]["k"], copies[0]["v"], copies[0]["logits"]))
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws_attn = torch.zeros(dreams.tree_verify_attn_workspace_size(copies[0]["kv"], copies[0]["tree"], w.Hq),
+                          dtype=torch.uint8, device=dev)
+    ws_step = torch.zeros(dreams.verify_step_workspace_size(copies[0]["tree"], w.V), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(c, ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        dreams.tree_verify_attn(c["q"], c["kv"], c["tree"], w.scale, out=c["out"],
+                                workspace=ws_attn if ws_attn.numel() else None, status=status)
+        if ev is not None:
+            ev[1].record(stream)
+        dreams.verify_step(c["logits"], c["tree"], c["kv"], max_path, outputs=c["outs"],
+                           workspace=ws_step, status=status)
+        if ev is not None:
+            ev[2].record(stream)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(max(3, args.warmup)):
+        step(copies[i % 2])
+    torch.cuda.synchronize(dev)
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item()):#x} on valid input")
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    t_load = time.time()  # keep the GPU busy ~1 s so the sampler sees the clocks under this load
+    while time.time() - t_load < 1.0:
+        for i in range(20):
+            step(copies[i % 2])
+        torch.cuda.synchronize(dev)
+
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    barrier()
+    t0 = time.time()
+    for i in range(K):
+        step(copies[i % 2], evs[i])
+    barrier()
+    wall = time.time() - t0
+    clk = clocks.stop()
+
+    total_ms = evs[0][0].elapsed_time(evs[-1][2])
+    attn_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    tail_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    ms_per_step = total_ms / K
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms_per_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_per_step = float(t.item())
+
+    # ---- e2e through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        c = copies[0]
+        host_in = {n: c[n].cpu().pin_memory() for n in ("q", "logits", "parent", "tokens", "tree_len", "kv_len")}
+        host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (c["outs"][0], c["outs"][2],
+                                                                             c["outs"][3])]
+        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        d2h = sum(t.numel() * t.element_size() for t in host_out)
+
+        def e2e_step():
+            for n, t in host_in.items():
+                c[n].copy_(t, non_blocking=True)
+            step(c)
+            for h, d in zip(host_out, (c["outs"][0], c["outs"][2], c["outs"][3])):
+                h.copy_(d, non_blocking=True)
+            stream.synchronize()
+
+        for _ in range(3):
+            e2e_step()
+        Ke = max(3, min(K, 50))
+        barrier()
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        s1.record(stream)
+        barrier()
+        e2e_us = s0.elapsed_time(s1) / Ke * 1000.0
+        e2e = {"value": round(e2e_us, 2), "unit": "us", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    ab, gb = attn_bytes(w), argmax_bytes(w)
+    attn_avg_ms = sum(attn_ms) / K
+    tail_avg_ms = sum(tail_ms) / K
+    peak, peak_kind = peaks()
+    achieved = ab / (attn_avg_ms * 1e-3) / 1e9
+    roofline = {
+        "kernel": "tree_attn (dreams_tree_verify_attn)",
+        "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+        "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+        "frac_of_nominal_8000": round(achieved / NOMINAL_HBM_GBS, 4),
+        "algorithmic_bytes": ab, "avg_launch_us": round(attn_avg_ms * 1000, 2),
+        "traffic": None,
+    }
+    tail_gbs = gb / (tail_avg_ms * 1e-3) / 1e9
+    kernels = {
+        "tree_attn": {"us": round(attn_avg_ms * 1000, 2), "bytes": ab, "GBps": round(achieved, 1),
+                      "frac_measured_hbm": round(achieved / peak, 4),
+                      "tflops": round(attn_flops(w) / (attn_avg_ms * 1e-3) / 1e12, 1)},
+        "verify_step": {"us": round(tail_avg_ms * 1000, 2), "argmax_bytes": gb, "GBps": round(tail_gbs, 1),
+                        "frac_measured_hbm": round(tail_gbs / peak, 4)},
+    }
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": "verify-step us (tree attention + argmax/accept/compaction)",
+            "value": round(ms_per_step * 1000.0, 2), "unit": "us", "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; shapes of the paper's VLM decoding workloads)",
+            "config": {"workload": w.spec.description, "name": w.spec.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv,
+                       "D": w.D, "T_max": w.T_max, "V": w.V, "logits": w.logits_dtype,
+                       "kv_tokens": int((w.kv_len + w.tree_len).sum()), "tree_nodes": int(w.tree_len.sum()),
+                       "l2": f"inputs larger than L2: 2 rotating copies of {copy_bytes / 2**20:.0f} MiB each",
+                       "parallelism": f"replicas x{world}"},
+            "e2e": e2e, "gpu_launches": 2 * K, "roofline": roofline, "kernels": kernels,
+            "tau_mean_accept_len": None, "clocks": clk, "cpu_baseline": cpu, "wall_s": round(wall, 3),
+        }
+        acc = copies[0]["outs"][0].float().mean().item()
+        line["tau_mean_accept_len"] = round(acc, 3)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_predictions(w: W.Workload) -> np.ndarray:
+    """The oracle's argmax of every logits row (computed once, untimed, so the
+    timed acceptance and compaction see the workload's real accepted paths)."""
+    import oracle
+    x = w.logits.reshape(-1, w.V)
+    am = oracle.argmax(W.bits(x), bf16_bits=True) if w.logits_dtype == "bf16" else oracle.argmax(x.numpy())
+    return am.reshape(w.B, w.T_max)
+
+
+def oracle_step_sample(w: W.Workload, rng, attn_rows: int, argmax_rows: int, am_all: np.ndarray):
+    """Runs the oracle on a sample of one step; returns (seconds scaled to a
+    full step, description, seconds spent)."""
+    import oracle
+    lay = (oracle.KVLayout(w.capacity, w.Hkv, w.D, page_table=w.page_table.numpy(), page_size=w.page_size,
+                           num_pages=w.num_pages) if w.paged else oracle.KVLayout(w.capacity, w.Hkv, w.D))
+    all_rows = np.array([(b, t, h) for b in range(w.B) for t in range(int(w.tree_len[b])) for h in range(w.Hq)],
+                        np.int32)
+    sel = all_rows[rng.choice(len(all_rows), min(attn_rows, len(all_rows)), replace=False)]
+    qb, kb, vb = W.bits(w.q), W.bits(w.k), W.bits(w.v)
+    t0 = time.perf_counter()
+    oracle.tree_attention(qb, kb, vb, lay, w.parent.numpy(), w.tree_len.numpy(), w.kv_len.numpy(), w.Hq, w.scale,
+                          sel=sel)
+    t_attn = time.perf_counter() - t0
+    valid = np.array([(b, i) for b in range(w.B) for i in range(int(w.tree_len[b]))])
+    pick = valid[rng.choice(len(valid), min(argmax_rows, len(valid)), replace=False)]
+    rows = w.logits[pick[:, 0], pick[:, 1]]
+    t0 = time.perf_counter()
+    if w.logits_dtype == "bf16":
+        oracle.argmax(W.bits(rows), bf16_bits=True)
+    else:
+        oracle.argmax(rows.numpy())
+    t_am = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    r = oracle.accept_path(am_all, w.parent.numpy(), w.tokens.numpy(), w.tree_len.numpy(), w.kv_len.numpy(),
+                           w.max_path)
+    oracle.kv_compact(kb, vb, lay, w.kv_len.numpy(), r["accept_len"], r["path"])
+    t_tail = time.perf_counter() - t0
+    full = t_attn * len(all_rows) / len(sel) + t_am * len(valid) / len(pick) + t_tail
+    desc = (f"{len(sel)} of {len(all_rows)} attention rows, {len(pick)} of {len(valid)} argmax rows, "
+            f"full acceptance + compaction; scaled to one full step")
+    return full, desc, t_attn + t_am + t_tail
+
+
+def cpu_baseline(w: W.Workload, budget_s: float):
+    rng = np.random.default_rng(0)
+    am_all = oracle_predictions(w)
+    # calibrate the attention cost per row, then size the sample to the budget
+    _, _, t = oracle_step_sample(w, rng, 16, 4, am_all)
+    per_row = max(t, 1e-3) / 16
+    rows = int(max(64, min(budget_s / per_row, 1 << 20)))
+    full_s, desc, spent = oracle_step_sample(w, rng, rows, max(8, rows // 64), am_all)
+    return {"value": round(full_s * 1e6, 1), "unit": "us", "cores": 1, "kind": "oracle",
+            "sample": desc + f" ({spent:.1f} s of CPU work; host has {os.cpu_count()} cores, 1 used)"}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    w = W.make(args.config)
+    rng = np.random.default_rng(1)
+    am_all = oracle_predictions(w)
+    for _ in range(args.warmup):
+        oracle_step_sample(w, rng, 16, 4, am_all)
+    vals, descs, spent = [], None, 0.0
+    t0 = time.time()
+    for _ in range(args.steps):
+        v, descs, s = oracle_step_sample(w, rng, 128, 16, am_all)
+        vals.append(v)
+        spent += s
+    wall = time.time() - t0
+    us = statistics.mean(vals) * 1e6
+    line = {
+        "metric": "verify-step us (tree attention + argmax/accept/compaction)", "impl": "reference",
+        "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(us / 1000, 3), "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic (seeded; shapes of the paper's VLM decoding workloads)",
+        "config": {"workload": w.spec.description, "name": w.spec.name},
+        "cpu_baseline": {"value": round(us, 1), "unit": "us", "cores": 1, "kind": "oracle",
+                         "sample": f"per step: {descs} (host has {os.cpu_count()} cores, 1 used)"},
+        "e2e": {"value": round(us, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0, "wall_s": round(wall, 2),
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_dreams(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,210 @@
+/*
+ * dreams.h -- C ABI of the GB300 (sm_103a) library for the target model's
+ * tree verification step of DREAM-S speculative decoding for vision-language
+ * models (arXiv 2606.00535).
+ *
+ * One verification step (paper Sec. 2, "Speculative decoding"): the target
+ * model scores every draft token in one parallel pass, then accepts drafts in
+ * order while they equal its own prediction, replacing the first mismatch by
+ * its own token. Here the drafts form a tree (parent array), so the step is
+ *
+ *   1. dreams_tree_verify_attn  tree-masked attention of the T tree tokens
+ *                               against the image-plus-text KV cache (Sec. 2,
+ *                               "Vision-Language Models": every cached visual
+ *                               and text token takes part in attention at each
+ *                               decoding step), once per layer;
+ *   2. dreams_vocab_argmax      the target's greedy prediction per tree node
+ *                               (temperature 0, Table 2);
+ *   3. dreams_accept_path       the longest root path whose drafts match, plus
+ *                               the target's bonus token;
+ *   4. dreams_kv_compact        the accepted nodes' K/V moved into contiguous
+ *                               cache slots for the next step;
+ *   5. dreams_verify_step       2 + 3 + 4 in one launch.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All data pointers are DEVICE pointers owned by the caller; the library
+ *    allocates no memory. Scratch comes from a caller-supplied workspace
+ *    whose size the matching *_workspace_size function returns. A workspace
+ *    must be zero-filled once when it is allocated; every call leaves it
+ *    zero-filled again (its counters reset themselves), so it can be reused
+ *    by later calls on the same stream. Calls that overlap in time must not
+ *    share a workspace.
+ *  - Every call is asynchronous on the given stream (NULL = the legacy
+ *    default stream) and runs on the current CUDA device.
+ *  - Host-side checks (null pointers, sizes, alignment, supported shapes)
+ *    run before any launch. A failed check returns DREAMS_ERR_INVALID_ARG or
+ *    DREAMS_ERR_UNSUPPORTED and launches nothing.
+ *  - Malformed device data (a bad parent array, tree or cache length, page
+ *    id or path) is never trapped: the kernels OR a DREAMS_DATA_* bit into
+ *    *status_word (a device int32, may be NULL) and skip the affected
+ *    sequence, whose outputs are then as documented per call.
+ *  - A launch failure returns DREAMS_ERR_CUDA; dreams_last_cuda_error()
+ *    gives the CUDA error code of the calling thread's last failure.
+ *
+ * Shapes (B sequences; T_max tree nodes per sequence including the root;
+ * Hq query heads; Hkv KV heads with Hq % Hkv == 0; head dim D in {64, 128}):
+ *  - tree node 0 is the root: the last committed token, whose K/V this pass
+ *    has just written to cache slot kv_len[b]; node i sits in slot
+ *    kv_len[b] + i. parent[b][0] = -1 and 0 <= parent[b][i] < i.
+ */
+#ifndef DREAMS_H_
+#define DREAMS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DREAMS_VERSION 10000 /* 1.0.0 */
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *dreams_stream_t;
+
+typedef enum dreams_status {
+  DREAMS_OK = 0,
+  DREAMS_ERR_INVALID_ARG = 1, /* null pointer, bad size, misaligned pointer */
+  DREAMS_ERR_UNSUPPORTED = 2, /* valid but unsupported shape or dtype */
+  DREAMS_ERR_WORKSPACE = 3,   /* workspace missing or too small */
+  DREAMS_ERR_CUDA = 4         /* a CUDA call failed; see dreams_last_cuda_error */
+} dreams_status_t;
+
+typedef enum dreams_dtype { DREAMS_F32 = 0, DREAMS_BF16 = 1 } dreams_dtype_t;
+
+/* Bits OR-ed into *status_word by the kernels. */
+#define DREAMS_DATA_BAD_PARENT 0x1   /* parent[0] != -1 or parent[i] outside [0, i) */
+#define DREAMS_DATA_BAD_TREE_LEN 0x2 /* tree_len outside [1, T_max] */
+#define DREAMS_DATA_BAD_KV_LEN 0x4   /* kv_len < 0 or kv_len + tree_len > capacity */
+#define DREAMS_DATA_BAD_PAGE 0x8     /* page-table entry outside [0, num_pages) */
+#define DREAMS_DATA_BAD_PATH 0x10    /* path[0] != 0 or not strictly increasing */
+
+/*
+ * One attention layer's K and V cache (bf16), or n_layers of them.
+ *  - contiguous (page_table == NULL): element (b, s, g, d) at
+ *        ((b * capacity + s) * Hkv + g) * D + d
+ *  - paged: logical slot s of sequence b is row s % page_size of physical
+ *    page p = page_table[b * pages_per_seq + s / page_size], and element
+ *    (b, s, g, d) is at ((p * page_size + s % page_size) * Hkv + g) * D + d;
+ *    capacity must equal pages_per_seq * page_size. Only page_size 64.
+ *  - layer l's cache starts layer_stride elements after layer l-1's (k and v
+ *    alike). k, v and layer_stride * 2 bytes must be 16-byte aligned.
+ */
+typedef struct dreams_kv_cache {
+  void *k;
+  void *v;
+  int32_t n_layers;
+  int64_t layer_stride;
+  int32_t Hkv;
+  int32_t D;
+  int32_t capacity;
+  const int32_t *page_table;
+  int32_t page_size;
+  int32_t pages_per_seq;
+  int32_t num_pages;
+} dreams_kv_cache_t;
+
+/* The draft trees of a batch (all device int32 arrays). */
+typedef struct dreams_tree {
+  const int32_t *parent;   /* [B, T_max] */
+  const int32_t *tokens;   /* [B, T_max] draft token ids; tokens[b][0] is never checked */
+  const int32_t *tree_len; /* [B] nodes in use, 1..T_max */
+  const int32_t *kv_len;   /* [B] committed prefix length L_b */
+  int32_t B;
+  int32_t T_max; /* 1..64 */
+} dreams_tree_t;
+
+/*
+ * Tree-masked verification attention for one layer (Sec. 2, "Speculative
+ * decoding" and "Vision-Language Models"; attention = softmax(Q K^T * scale)
+ * as in Sec. 3.2). For every sequence b, tree node t < tree_len[b] and query
+ * head h, with KV head g = h / (Hq / Hkv):
+ *     keys  J = { slots 0 .. L_b - 1 } U { slot L_b + a : a = t or an ancestor of t }
+ *     out[b, t, h, :] = sum_{j in J} softmax_j(scale * <q, K[b, j, g]>) V[b, j, g, :]
+ *     lse[b, t, h]    = log sum_{j in J} exp(scale * <q, K[b, j, g]>)
+ * q, out: bf16 [B, T_max, Hq, D] (16-byte aligned). lse: f32 [B, T_max, Hq]
+ * or NULL. Rows t >= tree_len[b] of out and lse are left untouched, and so are
+ * all rows of a sequence with bad data. layer selects the cache
+ * (0 <= layer < kv->n_layers). Accumulation is fp32; the output is rounded to
+ * bf16 once.
+ */
+size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
+                                              int32_t Hq);
+dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+                                        const dreams_tree_t *tree, int32_t Hq, float scale, void *out,
+                                        float *lse, void *workspace, size_t workspace_bytes,
+                                        int32_t *status_word, dreams_stream_t stream);
+
+/*
+ * Row-wise argmax (the target's greedy prediction, Sec. 2 "Speculative
+ * decoding" at temperature 0): out_idx[r] = argmax_v logits[r * row_stride + v]
+ * for v < V, under the total order "greater value wins, equal values (+0 ==
+ * -0) go to the lower index, NaN is above every number and the first NaN
+ * wins" -- the same result as torch.argmax. logits: f32 or bf16, rows x
+ * row_stride elements; row_stride >= V. Rows that start 16-byte aligned are
+ * read with 16-byte loads.
+ */
+size_t dreams_vocab_argmax_workspace_size(int64_t rows, int64_t V);
+dreams_status_t dreams_vocab_argmax(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
+                                    int64_t row_stride, int32_t *out_idx, void *workspace,
+                                    size_t workspace_bytes, dreams_stream_t stream);
+
+/*
+ * Greedy acceptance over the draft tree (Sec. 2 "Speculative decoding",
+ * generalised from a chain to a tree). argmax: [B, T_max] target predictions
+ * (row b * T_max + i is node i of sequence b). A root path 0 -> c1 -> ... -> cn
+ * matches when tokens[ck] == argmax[c(k-1)] for every k. The accepted path is
+ * the longest matching root path, cut to at most max_path - 1 drafts, ties to
+ * the lexicographically smallest node sequence. Outputs per sequence b:
+ *     path[b]       = (0, c1, ..., cn, -1, ...)                  [B, max_path]
+ *     out_tokens[b] = (tokens[c1], ..., tokens[cn], argmax[cn], -1, ...)
+ *     accept_len[b] = n + 1 (drafts plus the bonus token)
+ *     new_kv_len[b] = kv_len[b] + n + 1
+ * A sequence with a bad tree or kv_len < 0 gets accept_len 0, new_kv_len =
+ * kv_len and rows of -1. max_path >= 1.
+ */
+dreams_status_t dreams_accept_path(const int32_t *argmax, const dreams_tree_t *tree, int32_t max_path,
+                                   int32_t *accept_len, int32_t *path, int32_t *out_tokens,
+                                   int32_t *new_kv_len, int32_t *status_word, dreams_stream_t stream);
+
+/*
+ * KV compaction (keeps the cache a plain sequence for the next step, Sec. 2
+ * "Vision-Language Models"): for every sequence b with A = accept_len[b] > 0,
+ * every layer, K and V and every KV head,
+ *     slot L_b + x  <-  slot L_b + path[b][x]     for x = 0 .. A-1
+ * as if all A source rows were read before any is written. All other bytes are
+ * unchanged. path: [B, max_path], as returned by dreams_accept_path
+ * (path[b][0] = 0, strictly increasing); a sequence whose path is not of that
+ * form, or whose slots fall outside the capacity or on a bad page, is left
+ * untouched and flagged. kv->Hkv, kv->D give the head shape.
+ */
+dreams_status_t dreams_kv_compact(const dreams_kv_cache_t *kv, int32_t B, const int32_t *kv_len,
+                                  const int32_t *accept_len, const int32_t *path, int32_t max_path,
+                                  int32_t *status_word, dreams_stream_t stream);
+
+/*
+ * The verification tail in one launch: dreams_vocab_argmax over the rows of
+ * tree nodes (row b * T_max + i for i < tree_len[b]; logits [B, T_max, V]
+ * with row_stride), then dreams_accept_path, then dreams_kv_compact on all
+ * kv->n_layers layers, with the semantics documented above. argmax_out
+ * ([B, T_max], may be NULL) receives the predictions of the rows computed;
+ * other rows are untouched.
+ */
+size_t dreams_verify_step_workspace_size(const dreams_tree_t *tree, int64_t V);
+dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int64_t V,
+                                   int64_t row_stride, const dreams_tree_t *tree,
+                                   const dreams_kv_cache_t *kv, int32_t max_path, int32_t *argmax_out,
+                                   int32_t *accept_len, int32_t *path, int32_t *out_tokens,
+                                   int32_t *new_kv_len, void *workspace, size_t workspace_bytes,
+                                   int32_t *status_word, dreams_stream_t stream);
+
+const char *dreams_status_string(dreams_status_t status);
+int32_t dreams_version(void);
+int32_t dreams_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DREAMS_H_ */

@@ -1,0 +1,328 @@
+"""GB300 (sm_103a) tree verification for DREAM-S speculative decoding.
+
+A thin binding over the C ABI of ``libdreams.so`` (declared in
+``include/dreams.h``): each function checks the dtype, device and layout of
+its torch tensors, passes their ``data_ptr()`` and the current CUDA stream to
+the C entry point of the same name, and raises on a non-OK status. Every
+step of the computation runs in the library's CUDA kernels; there is no CPU
+or PyTorch fallback, and importing this package on a machine without the
+built library raises.
+
+The step it implements (paper Sec. 2, "Speculative decoding"): the target
+model scores all draft tokens in one pass, then accepts drafts while they
+equal its own greedy prediction; here the drafts form a tree.
+
+    out, lse = tree_verify_attn(q, kv, tree, scale)          # per layer
+    res = verify_step(logits, tree, kv, max_path)            # argmax + walk + compaction
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+from dataclasses import dataclass
+from typing import Dict, Optional, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdreams.so")
+HEADER = os.path.join(os.path.dirname(_HERE), "include", "dreams.h")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+F32, BF16 = 0, 1
+DATA_BAD_PARENT, DATA_BAD_TREE_LEN, DATA_BAD_KV_LEN, DATA_BAD_PAGE, DATA_BAD_PATH = 1, 2, 4, 8, 16
+
+
+class DreamsError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        msg = _lib().dreams_status_string(status).decode()
+        if status == ERR_CUDA:
+            msg += f" (cudaError {_lib().dreams_last_cuda_error()})"
+        super().__init__(f"{fn}: {msg}")
+        self.status = status
+
+
+class _KVCache(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("n_layers", ctypes.c_int32),
+                ("layer_stride", ctypes.c_int64), ("Hkv", ctypes.c_int32), ("D", ctypes.c_int32),
+                ("capacity", ctypes.c_int32), ("page_table", ctypes.c_void_p),
+                ("page_size", ctypes.c_int32), ("pages_per_seq", ctypes.c_int32),
+                ("num_pages", ctypes.c_int32)]
+
+
+class _Tree(ctypes.Structure):
+    _fields_ = [("parent", ctypes.c_void_p), ("tokens", ctypes.c_void_p), ("tree_len", ctypes.c_void_p),
+                ("kv_len", ctypes.c_void_p), ("B", ctypes.c_int32), ("T_max", ctypes.c_int32)]
+
+
+_LIB: Optional[ctypes.CDLL] = None
+_LOCK = threading.Lock()
+
+
+def _lib() -> ctypes.CDLL:
+    global _LIB
+    if _LIB is None:
+        with _LOCK:
+            if _LIB is None:
+                if not os.path.exists(LIB_PATH):
+                    raise ImportError(f"libdreams.so is not built ({LIB_PATH}); run "
+                                      "`python -c 'import __graft_entry__ as g; g.build()'`")
+                lib = ctypes.CDLL(LIB_PATH)
+                p, i32, i64, sz, f32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t,
+                                        ctypes.c_float)
+                pkv, ptr = ctypes.POINTER(_KVCache), ctypes.POINTER(_Tree)
+                sig = {
+                    "dreams_tree_verify_attn_workspace_size": (sz, [pkv, ptr, i32]),
+                    "dreams_tree_verify_attn": (ctypes.c_int, [p, pkv, i32, ptr, i32, f32, p, p, p, sz, p, p]),
+                    "dreams_vocab_argmax_workspace_size": (sz, [i64, i64]),
+                    "dreams_vocab_argmax": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p, sz, p]),
+                    "dreams_accept_path": (ctypes.c_int, [p, ptr, i32, p, p, p, p, p, p]),
+                    "dreams_kv_compact": (ctypes.c_int, [pkv, i32, p, p, p, i32, p, p]),
+                    "dreams_verify_step_workspace_size": (sz, [ptr, i64]),
+                    "dreams_verify_step": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, p, p, p, p,
+                                                          p, p, sz, p, p]),
+                    "dreams_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+                    "dreams_version": (i32, []),
+                    "dreams_last_cuda_error": (i32, []),
+                }
+                for name, (res, args) in sig.items():
+                    fn = getattr(lib, name)
+                    fn.restype = res
+                    fn.argtypes = args
+                _LIB = lib
+    return _LIB
+
+
+def declared_functions() -> list:
+    """Names of the functions ``include/dreams.h`` declares."""
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]*?\b(dreams_\w+)\s*\(", text, re.M)))
+
+
+def version() -> int:
+    return int(_lib().dreams_version())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(name: str, st: int):
+    if st != OK:
+        raise DreamsError(name, st)
+
+
+def _need(t: torch.Tensor, name: str, dtype, dev) -> torch.Tensor:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if t.device != dev:
+        raise ValueError(f"{name} must be on {dev}, got {t.device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+@dataclass
+class KVCache:
+    """K/V cache of one or more layers (bf16).
+
+    Contiguous: ``k, v`` of shape ``[B, capacity, Hkv, D]`` (one layer) or
+    ``[n_layers, B, capacity, Hkv, D]``. Paged: ``[num_pages, 64, Hkv, D]``
+    (or with a leading layer dim) plus ``page_table`` int32 ``[B, pages_per_seq]``.
+    """
+    k: torch.Tensor
+    v: torch.Tensor
+    page_table: Optional[torch.Tensor] = None
+
+    def __post_init__(self):
+        if self.k.shape != self.v.shape:
+            raise ValueError("k and v shapes differ")
+        dev = self.k.device
+        _need(self.k, "k", torch.bfloat16, dev)
+        _need(self.v, "v", torch.bfloat16, dev)
+        nd = self.k.dim()
+        if nd not in (4, 5):
+            raise ValueError("k must be 4-D or 5-D")
+        self.n_layers = self.k.shape[0] if nd == 5 else 1
+        shp = self.k.shape[1:] if nd == 5 else self.k.shape
+        self.layer_stride = int(shp.numel()) if nd == 5 else 0
+        self.Hkv, self.D = int(shp[2]), int(shp[3])
+        if self.page_table is None:
+            self.B = int(shp[0])
+            self.capacity = int(shp[1])
+            self.page_size = self.pages_per_seq = self.num_pages = 0
+        else:
+            _need(self.page_table, "page_table", torch.int32, dev)
+            self.B = int(self.page_table.shape[0])
+            self.page_size = int(shp[1])
+            self.pages_per_seq = int(self.page_table.shape[1])
+            self.num_pages = int(shp[0])
+            self.capacity = self.pages_per_seq * self.page_size
+        self._c = _KVCache(self.k.data_ptr(), self.v.data_ptr(), self.n_layers, self.layer_stride, self.Hkv,
+                           self.D, self.capacity,
+                           None if self.page_table is None else self.page_table.data_ptr(),
+                           self.page_size, self.pages_per_seq, self.num_pages)
+
+
+@dataclass
+class Tree:
+    """Draft trees of a batch: int32 ``parent``, ``tokens`` [B, T_max];
+    ``tree_len``, ``kv_len`` [B] (all on the same CUDA device)."""
+    parent: torch.Tensor
+    tokens: torch.Tensor
+    tree_len: torch.Tensor
+    kv_len: torch.Tensor
+
+    def __post_init__(self):
+        dev = self.parent.device
+        for n in ("parent", "tokens", "tree_len", "kv_len"):
+            _need(getattr(self, n), n, torch.int32, dev)
+        self.B, self.T_max = (int(x) for x in self.parent.shape)
+        if tuple(self.tokens.shape) != (self.B, self.T_max) or self.tree_len.numel() != self.B or \
+                self.kv_len.numel() != self.B:
+            raise ValueError("tree tensor shapes disagree")
+        self._c = _Tree(self.parent.data_ptr(), self.tokens.data_ptr(), self.tree_len.data_ptr(),
+                        self.kv_len.data_ptr(), self.B, self.T_max)
+
+
+# Zero-filled workspaces, one per (function, device, stream); the kernels
+# leave them zero-filled after each call.
+_WS: Dict[Tuple[str, int, int], torch.Tensor] = {}
+
+
+def _workspace(kind: str, nbytes: int, device: torch.device, stream) -> Optional[torch.Tensor]:
+    if nbytes == 0:
+        return None
+    key = (kind, device.index if device.index is not None else torch.cuda.current_device(),
+           (torch.cuda.current_stream(device) if stream is None else stream).cuda_stream)
+    ws = _WS.get(key)
+    if ws is None or ws.numel() < nbytes:
+        ws = torch.zeros(nbytes, dtype=torch.uint8, device=device)
+        _WS[key] = ws
+    return ws
+
+
+def tree_verify_attn_workspace_size(kv: KVCache, tree: Tree, Hq: int) -> int:
+    return int(_lib().dreams_tree_verify_attn_workspace_size(ctypes.byref(kv._c), ctypes.byref(tree._c), Hq))
+
+
+def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, layer: int = 0,
+                     out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
+                     want_lse: bool = False, workspace: Optional[torch.Tensor] = None,
+                     status: Optional[torch.Tensor] = None, stream=None):
+    """Tree-masked attention of the tree tokens' queries ``q`` (bf16
+    [B, T_max, Hq, D]) over the cache. Returns (out, lse or None)."""
+    dev = q.device
+    _need(q, "q", torch.bfloat16, dev)
+    Hq = int(q.shape[2])
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, dev)
+    if lse is None and want_lse:
+        lse = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
+    if lse is not None:
+        _need(lse, "lse", torch.float32, dev)
+    need = tree_verify_attn_workspace_size(kv, tree, Hq)
+    if workspace is None:
+        workspace = _workspace("attn", need, dev, stream)
+    st = _lib().dreams_tree_verify_attn(
+        _ptr(q), ctypes.byref(kv._c), layer, ctypes.byref(tree._c), Hq, float(scale), _ptr(out), _ptr(lse),
+        _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
+        _ptr(status), _stream(stream))
+    _check("dreams_tree_verify_attn", st)
+    return out, lse
+
+
+def vocab_argmax(logits: torch.Tensor, out: Optional[torch.Tensor] = None,
+                 workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Row-wise argmax of a 2-D (or flattened leading dims) f32 / bf16 tensor."""
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    V = int(logits.shape[-1])
+    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
+    if x.stride(-1) != 1:
+        raise ValueError("logits rows must be contiguous")
+    rows = int(x.shape[0])
+    if out is None:
+        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=logits.device)
+    _need(out, "out", torch.int32, logits.device)
+    need = int(_lib().dreams_vocab_argmax_workspace_size(rows, V))
+    if workspace is None:
+        workspace = _workspace("argmax", need, logits.device, stream)
+    st = _lib().dreams_vocab_argmax(
+        _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), _ptr(out),
+        _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
+    _check("dreams_vocab_argmax", st)
+    return out
+
+
+def _walk_outputs(B: int, max_path: int, dev):
+    return (torch.empty(B, dtype=torch.int32, device=dev),
+            torch.empty((B, max_path), dtype=torch.int32, device=dev),
+            torch.empty((B, max_path), dtype=torch.int32, device=dev),
+            torch.empty(B, dtype=torch.int32, device=dev))
+
+
+def accept_path(argmax: torch.Tensor, tree: Tree, max_path: int, status: Optional[torch.Tensor] = None,
+                stream=None) -> dict:
+    """Greedy acceptance over the trees. Returns a dict of device tensors."""
+    dev = tree.parent.device
+    _need(argmax, "argmax", torch.int32, dev)
+    acc, path, toks, nkl = _walk_outputs(tree.B, max_path, dev)
+    st = _lib().dreams_accept_path(_ptr(argmax), ctypes.byref(tree._c), max_path, _ptr(acc), _ptr(path),
+                                   _ptr(toks), _ptr(nkl), _ptr(status), _stream(stream))
+    _check("dreams_accept_path", st)
+    return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
+
+
+def kv_compact(kv: KVCache, kv_len: torch.Tensor, accept_len: torch.Tensor, path: torch.Tensor,
+               status: Optional[torch.Tensor] = None, stream=None) -> None:
+    """Moves the accepted slots into place, in all layers of ``kv``."""
+    dev = kv.k.device
+    for n, t in (("kv_len", kv_len), ("accept_len", accept_len), ("path", path)):
+        _need(t, n, torch.int32, dev)
+    B, max_path = (int(x) for x in path.shape)
+    st = _lib().dreams_kv_compact(ctypes.byref(kv._c), B, _ptr(kv_len), _ptr(accept_len), _ptr(path), max_path,
+                                  _ptr(status), _stream(stream))
+    _check("dreams_kv_compact", st)
+
+
+def verify_step_workspace_size(tree: Tree, V: int) -> int:
+    return int(_lib().dreams_verify_step_workspace_size(ctypes.byref(tree._c), V))
+
+
+def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
+                argmax_out: Optional[torch.Tensor] = None, outputs: Optional[tuple] = None,
+                workspace: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+                stream=None) -> dict:
+    """Argmax of the tree rows of ``logits`` ([B, T_max, V] f32/bf16), greedy
+    acceptance and KV compaction, in one launch."""
+    dev = tree.parent.device
+    if logits.dtype not in (torch.float32, torch.bfloat16) or logits.device != dev:
+        raise TypeError("logits must be float32/bfloat16 on the tree's device")
+    if logits.dim() != 3 or tuple(logits.shape[:2]) != (tree.B, tree.T_max) or logits.stride(-1) != 1 or \
+            logits.stride(0) != logits.shape[1] * logits.stride(1):
+        raise ValueError("logits must be [B, T_max, V] with uniformly strided contiguous rows")
+    V = int(logits.shape[2])
+    if argmax_out is not None:
+        _need(argmax_out, "argmax_out", torch.int32, dev)
+    acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
+    need = verify_step_workspace_size(tree, V)
+    if workspace is None:
+        workspace = _workspace("step", need, dev, stream)
+    st = _lib().dreams_verify_step(
+        _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
+        ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, _ptr(argmax_out), _ptr(acc), _ptr(path),
+        _ptr(toks), _ptr(nkl), _ptr(workspace), 0 if workspace is None else workspace.numel(), _ptr(status),
+        _stream(stream))
+    _check("dreams_verify_step", st)
+    return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}

@@ -1,0 +1,116 @@
+"""The C ABI on the CPU: the library builds for sm_103a, loads, exports every
+function include/dreams.h declares, and rejects bad arguments on the host
+before any launch. No compute runs here."""
+import ctypes
+import os
+import subprocess
+import sys
+
+import pytest
+import torch
+
+import paper_2606_00535_gb300 as dreams
+from paper_2606_00535_gb300 import build as libbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    libbuild.build()
+    return dreams._lib()
+
+
+def test_exports_every_declared_function(lib):
+    names = dreams.declared_functions()
+    assert len(names) == 11
+    for n in names:
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", dreams.LIB_PATH], capture_output=True, text=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    assert set(names) <= exported
+
+
+def test_version_and_strings(lib):
+    assert dreams.version() == 10000
+    for code, text in [(0, b"ok"), (1, b"invalid argument"), (3, b"workspace missing or too small"),
+                       (99, b"unknown status")]:
+        assert lib.dreams_status_string(code) == text
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    code = ("import paper_2606_00535_gb300 as d; d.LIB_PATH='/nonexistent/libdreams.so'\n"
+            "try:\n    d._lib()\nexcept ImportError as e:\n    print('raised', e)\n")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True)
+    assert "raised" in r.stdout
+
+
+def test_workspace_sizes(lib):
+    k = torch.empty(0, dtype=torch.bfloat16)
+    kvc = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
+    tr = dreams._Tree(16, 16, 16, 16, 16, 64)
+    n = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32)
+    assert n > 0 and n % 256 == 0
+    bad = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(bad), ctypes.byref(tr), 30) == 0
+    assert lib.dreams_vocab_argmax_workspace_size(768, 128256) >= 0
+    assert lib.dreams_verify_step_workspace_size(ctypes.byref(tr), 128256) >= 16 * 64 * 16
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="host-validation cases use placeholder pointers")
+def test_invalid_arguments_rejected_before_launch(lib):
+    """Each case breaks exactly one rule and must be refused on the host."""
+    P = 0x1000  # placeholder, never dereferenced: every call below fails validation
+    null = None
+    tr = dreams._Tree(P, P, P, P, 2, 8)
+    kvc = dreams._KVCache(P, P, 1, 0, 2, 128, 256, None, 0, 0, 0)
+    st = ctypes.c_void_p(P)
+    s = ctypes.c_void_p(0)
+
+    def attn(q=P, kv=kvc, layer=0, tree=tr, Hq=4, scale=0.1, out=P, ws=None, wsb=0):
+        return lib.dreams_tree_verify_attn(q, ctypes.byref(kv), layer, ctypes.byref(tree), Hq, scale, out, null,
+                                           ws, wsb, st, s)
+
+    assert attn(q=null) == dreams.ERR_INVALID_ARG
+    assert attn(out=null) == dreams.ERR_INVALID_ARG
+    assert attn(q=P + 2) == dreams.ERR_INVALID_ARG           # misaligned
+    assert attn(Hq=3) == dreams.ERR_INVALID_ARG              # Hq % Hkv
+    assert attn(layer=1) == dreams.ERR_INVALID_ARG
+    assert attn(scale=float("inf")) == dreams.ERR_INVALID_ARG
+    assert attn(tree=dreams._Tree(P, P, P, P, 2, 65)) == dreams.ERR_INVALID_ARG   # T_max > 64
+    assert attn(tree=dreams._Tree(P, P, P, P, 0, 8)) == dreams.ERR_INVALID_ARG
+    assert attn(kv=dreams._KVCache(P, P, 1, 0, 2, 96, 256, None, 0, 0, 0)) == dreams.ERR_UNSUPPORTED
+    assert attn(kv=dreams._KVCache(P, P, 1, 0, 2, 128, 256, P, 32, 8, 4)) == dreams.ERR_UNSUPPORTED
+    assert attn(kv=dreams._KVCache(P, P, 1, 0, 2, 128, 256, P, 64, 5, 4)) == dreams.ERR_INVALID_ARG
+    big = dreams._KVCache(P, P, 1, 0, 1, 128, 100000, None, 0, 0, 0)
+    need = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(big), ctypes.byref(tr), 1)
+    assert need > 0
+    assert attn(kv=big, Hq=1, ws=None, wsb=0) == dreams.ERR_WORKSPACE
+    assert attn(kv=big, Hq=1, ws=P, wsb=need - 1) == dreams.ERR_WORKSPACE
+
+    am = lib.dreams_vocab_argmax
+    assert am(null, 0, 4, 100, 100, P, null, 0, s) == dreams.ERR_INVALID_ARG
+    assert am(P, 0, 4, 100, 99, P, null, 0, s) == dreams.ERR_INVALID_ARG     # stride < V
+    assert am(P, 7, 4, 100, 100, P, null, 0, s) == dreams.ERR_UNSUPPORTED
+    assert am(P + 1, 1, 4, 100, 100, P, null, 0, s) == dreams.ERR_INVALID_ARG  # misaligned bf16
+    assert am(P, 0, 1, 10_000_000, 10_000_000, P, null, 0, s) == dreams.ERR_WORKSPACE
+
+    ap = lib.dreams_accept_path
+    assert ap(P, ctypes.byref(tr), 0, P, P, P, P, st, s) == dreams.ERR_INVALID_ARG
+    assert ap(P, ctypes.byref(dreams._Tree(P, null, P, P, 2, 8)), 4, P, P, P, P, st, s) == dreams.ERR_INVALID_ARG
+    assert ap(null, ctypes.byref(tr), 4, P, P, P, P, st, s) == dreams.ERR_INVALID_ARG
+
+    kc = lib.dreams_kv_compact
+    assert kc(ctypes.byref(kvc), 0, P, P, P, 4, st, s) == dreams.ERR_INVALID_ARG
+    assert kc(ctypes.byref(kvc), 2, P, P, P, 66, st, s) == dreams.ERR_INVALID_ARG
+    assert kc(ctypes.byref(dreams._KVCache(P + 8, P, 1, 0, 2, 128, 256, None, 0, 0, 0)), 2, P, P, P, 4, st,
+              s) == dreams.ERR_INVALID_ARG
+
+    vs = lib.dreams_verify_step
+    wsb = lib.dreams_verify_step_workspace_size(ctypes.byref(tr), 1000)
+    assert vs(P, 0, 1000, 1000, ctypes.byref(tr), ctypes.byref(kvc), 5, null, P, P, P, P, P, wsb - 1, st,
+              s) == dreams.ERR_WORKSPACE
+    assert vs(P, 0, 1000, 999, ctypes.byref(tr), ctypes.byref(kvc), 5, null, P, P, P, P, P, wsb, st,
+              s) == dreams.ERR_INVALID_ARG
+    assert vs(P, 3, 1000, 1000, ctypes.byref(tr), ctypes.byref(kvc), 5, null, P, P, P, P, P, wsb, st,
+              s) == dreams.ERR_UNSUPPORTED

@@ -1,0 +1,355 @@
+"""GPU parity: every kernel, through the C ABI, against the fp64 oracle on the
+same seeded inputs (bit-exact for indices, paths, tokens and the compacted
+cache; attention within max-abs 1e-2 / mean-abs 1e-3 and lse within 1e-3
+relative)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as W
+from helpers import compare_attention, layout, logits_rows_oracle, oracle_attention, to_gpu
+
+pytestmark = pytest.mark.gpu
+
+CONFIGS = ["tiny", "llava7b", "qwen2vl7b", "long13b", "batched"]
+
+
+@pytest.fixture(scope="module")
+def dreams():
+    import paper_2606_00535_gb300 as d
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    d._lib()  # fails loudly when the library is missing
+    return d
+
+
+def _status():
+    return torch.zeros(1, dtype=torch.int32, device="cuda")
+
+
+# ------------------------------------------------------------------ attention
+@pytest.mark.parametrize("name", CONFIGS)
+def test_attention_matches_oracle(dreams, name):
+    w = W.make(name, with_logits=False)
+    g = to_gpu(w)
+    st = _status()
+    out, lse = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    rng = np.random.default_rng(5)
+    if name == "batched":  # all heads of sampled nodes, plus every node of one sequence
+        sel = []
+        for b in range(w.B):
+            for t in rng.choice(int(w.tree_len[b]), 6, replace=False):
+                sel += [(b, int(t), h) for h in range(w.Hq)]
+        sel += [(3, t, h) for t in range(int(w.tree_len[3])) for h in (0, 13, 31)]
+        sel = np.array(sel, np.int32)
+    else:
+        sel = None
+    ref, ref_lse, sel, ost = oracle_attention(w, sel)
+    assert ost == 0
+    compare_attention(out, lse, ref, ref_lse, sel)
+
+
+@pytest.mark.parametrize("name,L,key_scale", [("tiny", 0, 1.0), ("tiny", 16, 8.0), ("llava7b", 16, 8.0),
+                                              ("qwen2vl7b", 0, 8.0), ("tiny", 300, 8.0)])
+def test_attention_mask_sensitive(dreams, name, L, key_scale):
+    """Short prefixes and tree keys scaled x8: the tree columns dominate, so a
+    wrong ancestor mask moves the output far outside the tolerance. The
+    dominated softmax makes |out| ~ |V| (<= ~4), so the bf16 rounding of the
+    output and of the probabilities gives up to ~2 * 2^-9 * 4 = 1.6e-2."""
+    w = W.make(name, with_logits=False, kv_len_override=L, tree_key_scale=key_scale)
+    g = to_gpu(w)
+    st = _status()
+    out, lse = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True, status=st)
+    ref, ref_lse, sel, _ = oracle_attention(w)
+    assert int(st.item()) == 0
+    compare_attention(out, lse, ref, ref_lse, sel, max_abs=2e-2, mean_abs=2e-3)
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,D,T,L,cap", [
+    (1, 1, 1, 64, 1, 0, 1),        # root only, empty prefix
+    (1, 2, 1, 128, 1, 5, 8),       # root only
+    (2, 8, 2, 128, 17, 63, 200),   # ragged tile boundary
+    (3, 4, 4, 64, 64, 129, 400),   # maximum tree
+    (2, 16, 2, 128, 64, 1000, 1100),  # 512 query rows per KV head: several row blocks
+])
+def test_attention_edge_shapes(dreams, B, Hq, Hkv, D, T, L, cap):
+    rng = np.random.default_rng(B * 1000 + T)
+    par = np.full((B, T), -1, np.int32)
+    for b in range(B):
+        par[b] = W.random_tree(rng, T)
+    tl = np.full(B, T, np.int32)
+    tl[-1] = max(1, T - 3)
+    par[-1, tl[-1]:] = -1
+    kl = rng.integers(max(0, L - 5), L + 1, B).astype(np.int32)
+    kl = np.minimum(kl, cap - tl)
+    q = W.bf16(rng.standard_normal((B, T, Hq, D), dtype=np.float32))
+    k = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    v = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    scale = 1.0 / np.sqrt(D)
+    kv = dreams.KVCache(k.cuda(), v.cuda())
+    tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
+                       torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    out = torch.full((B, T, Hq, D), 7.0, dtype=torch.bfloat16, device="cuda")
+    out, lse = dreams.tree_verify_attn(q.cuda(), kv, tree, scale, out=out, want_lse=True)
+    ref, ref_lse, sel, st = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v), oracle.KVLayout(cap, Hkv, D),
+                                                  par, tl, kl, Hq, scale)
+    assert st == 0
+    compare_attention(out, lse, ref, ref_lse, sel)
+    # rows past tree_len are untouched
+    assert (out[-1, tl[-1]:].float() == 7.0).all()
+
+
+def test_attention_paged_equals_contiguous(dreams):
+    """The batched workload copied into a contiguous cache gives bit-identical
+    results to its paged form."""
+    w = W.make("batched", with_logits=False)
+    g = to_gpu(w)
+    out_p, lse_p = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True)
+    pt = w.page_table.numpy()
+    cap = w.capacity
+    kc = torch.zeros((w.B, cap, w.Hkv, w.D), dtype=torch.bfloat16)
+    vc = torch.zeros_like(kc)
+    for b in range(w.B):
+        for j in range(w.pages_per_seq):
+            if pt[b, j] >= 0:
+                kc[b, j * 64:(j + 1) * 64] = w.k[pt[b, j]]
+                vc[b, j * 64:(j + 1) * 64] = w.v[pt[b, j]]
+    kv_c = dreams.KVCache(kc.cuda(), vc.cuda())
+    out_c, lse_c = dreams.tree_verify_attn(g["q"], kv_c, g["tree"], w.scale, want_lse=True)
+    for b in range(w.B):
+        t = int(w.tree_len[b])
+        assert torch.equal(out_p[b, :t], out_c[b, :t])
+        assert torch.equal(lse_p[b, :t], lse_c[b, :t])
+
+
+def test_attention_repeatable(dreams):
+    """Two calls on the same inputs give identical bits (the split merge has a
+    fixed order and the workspace counters reset themselves)."""
+    w = W.make("long13b", with_logits=False)
+    g = to_gpu(w)
+    a, la = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True)
+    a = a.clone()
+    la = la.clone()
+    b, lb = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True)
+    assert torch.equal(a, b) and torch.equal(la, lb)
+
+
+# ------------------------------------------------------------------ argmax
+@pytest.mark.parametrize("name", CONFIGS)
+def test_argmax_matches_oracle(dreams, name):
+    w = W.make(name, with_attn=False)
+    x = w.logits.cuda()
+    am = dreams.vocab_argmax(x)
+    ref = logits_rows_oracle(w)
+    np.testing.assert_array_equal(am.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_argmax_edge_rows(dreams, dtype):
+    nan, inf = float("nan"), float("inf")
+    V = 4099  # not a multiple of the vector width
+    rng = np.random.default_rng(9)
+    x = rng.standard_normal((12, V)).astype(np.float32)
+    x[0, :] = 1.0                   # all equal -> 0
+    x[1, [5, 4000]] = 50.0          # tie across chunks -> 5
+    x[2, :] = -0.0
+    x[2, 3000] = 0.0                # +0 == -0 -> 0
+    x[3, :] = -inf                  # -> 0
+    x[4, [17, 2000]] = nan          # first NaN -> 17
+    x[5, 4098] = 99.0               # tail element
+    x[6, 0] = inf
+    x[6, 1] = inf                   # -> 0
+    x[7, :] = -1.0
+    x[7, 4097] = -0.5               # tail
+    x[8, 3] = nan
+    x[8, 2] = inf                   # NaN beats inf -> 3
+    x[9, 4096:] = 1e30              # tail maxima, first wins
+    t = torch.from_numpy(x).to(dtype)
+    ref = (oracle.argmax(W.bits(t), bf16_bits=True) if dtype == torch.bfloat16 else oracle.argmax(x))
+    np.testing.assert_array_equal(dreams.vocab_argmax(t.cuda()).cpu().numpy(), ref)
+    np.testing.assert_array_equal(ref[:10], [0, 5, 0, 0, 17, 4098, 0, 4097, 3, 4096])
+    # padded rows (row_stride > V) and a base that is not 16-byte aligned
+    pad = torch.full((12, V + 5), 1e30, dtype=dtype)
+    pad[:, 1:V + 1] = t
+    got = dreams.vocab_argmax(pad.cuda()[:, 1:V + 1])
+    np.testing.assert_array_equal(got.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("rows,V", [(1, 1), (3, 7), (1, 152064), (700, 9), (2, 1_000_003)])
+def test_argmax_shapes(dreams, rows, V):
+    rng = np.random.default_rng(rows + V)
+    x = (rng.standard_normal((rows, V)) * 3).astype(np.float32)
+    t = torch.from_numpy(x).to(torch.bfloat16)
+    np.testing.assert_array_equal(dreams.vocab_argmax(t.cuda()).cpu().numpy(),
+                                  oracle.argmax(W.bits(t), bf16_bits=True))
+    np.testing.assert_array_equal(dreams.vocab_argmax(torch.from_numpy(x).cuda()).cpu().numpy(),
+                                  oracle.argmax(x))
+
+
+# ------------------------------------------------------------------ acceptance
+def _tree_gpu(dreams, parent, tokens, tree_len, kv_len):
+    f = lambda a: torch.as_tensor(np.asarray(a, np.int32)).cuda()
+    return dreams.Tree(f(parent), f(tokens), f(tree_len), f(kv_len))
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_accept_path_random_trees(dreams, seed):
+    rng = np.random.default_rng(seed)
+    B, T_max = 40, 64
+    par = np.full((B, T_max), -1, np.int32)
+    tl = rng.integers(1, T_max + 1, B).astype(np.int32)
+    for b in range(B):
+        par[b, :tl[b]] = W.random_tree(rng, int(tl[b]))
+    vocab = [2, 3, 5, 50][seed % 4]
+    tok = rng.integers(0, vocab, (B, T_max)).astype(np.int32)
+    am = rng.integers(0, vocab, (B, T_max)).astype(np.int32)
+    kl = rng.integers(0, 5000, B).astype(np.int32)
+    max_path = [65, 8, 3, 1, 30, 65][seed]
+    tree = _tree_gpu(dreams, par, tok, tl, kl)
+    r = dreams.accept_path(torch.from_numpy(am).cuda(), tree, max_path)
+    ref = oracle.accept_path(am, par, tok, tl, kl, max_path)
+    for key in ("accept_len", "path", "out_tokens", "new_kv_len"):
+        np.testing.assert_array_equal(r[key].cpu().numpy(), ref[key], err_msg=key)
+
+
+def test_accept_path_bad_data(dreams):
+    par = np.array([[-1, 0, 0, 1], [-1, 0, 2, 1], [0, 0, 1, 2], [-1, 0, 0, 0]], np.int32)
+    tl = np.array([4, 4, 4, 9], np.int32)
+    kl = np.array([3, 3, 3, 3], np.int32)
+    kl2 = np.array([-1, 3, 3, 3], np.int32)
+    tok = np.zeros((4, 4), np.int32)
+    am = np.zeros((4, 4), np.int32)
+    st = _status()
+    r = dreams.accept_path(torch.from_numpy(am).cuda(), _tree_gpu(dreams, par, tok, tl, kl2), 5, status=st)
+    s = int(st.item())
+    assert s & dreams.DATA_BAD_PARENT and s & dreams.DATA_BAD_TREE_LEN and s & dreams.DATA_BAD_KV_LEN
+    np.testing.assert_array_equal(r["accept_len"].cpu().numpy(), [0, 0, 0, 0])
+    np.testing.assert_array_equal(r["new_kv_len"].cpu().numpy(), kl2)
+    assert (r["path"].cpu().numpy() == -1).all()
+
+
+# ------------------------------------------------------------------ compaction
+@pytest.mark.parametrize("paged", [False, True])
+def test_kv_compact_matches_oracle(dreams, paged):
+    rng = np.random.default_rng(31 + paged)
+    B, cap, Hkv, D, n_layers, page = 5, 256, 4, 128, 3, 64
+    k = rng.integers(0, 65536, (n_layers, B, cap, Hkv, D), dtype=np.uint16)
+    v = rng.integers(0, 65536, (n_layers, B, cap, Hkv, D), dtype=np.uint16)
+    L = np.array([10, 0, 60, 100, 180], np.int32)
+    max_path = 9
+    acc = np.array([3, 1, 8, 0, 9], np.int32)
+    path = np.full((B, max_path), -1, np.int32)
+    path[0, :3] = [0, 2, 3]
+    path[1, :1] = [0]
+    path[2, :8] = [0, 1, 5, 7, 9, 10, 30, 63]
+    path[4, :9] = [0, 3, 4, 6, 8, 20, 40, 70, 75]
+    if paged:
+        pps = cap // page
+        table = rng.permutation(B * pps).astype(np.int32).reshape(B, pps)
+        kin = np.empty((n_layers, B * pps, page, Hkv, D), np.uint16)
+        vin = np.empty_like(kin)
+        for b in range(B):
+            for j in range(pps):
+                kin[:, table[b, j]] = k[:, b, j * page:(j + 1) * page]
+                vin[:, table[b, j]] = v[:, b, j * page:(j + 1) * page]
+        lay = oracle.KVLayout(cap, Hkv, D, page_table=table, page_size=page, num_pages=B * pps)
+        pt = torch.from_numpy(table).cuda()
+    else:
+        kin, vin, pt = k, v, None
+        lay = oracle.KVLayout(cap, Hkv, D)
+    ko, vo, ost = oracle.kv_compact(kin, vin, lay, L, acc, path, n_layers=n_layers,
+                                    layer_stride=kin[0].size)
+    assert ost == 0
+    tk = torch.from_numpy(kin.view(np.int16)).view(torch.bfloat16).cuda()
+    tv = torch.from_numpy(vin.view(np.int16)).view(torch.bfloat16).cuda()
+    kv = dreams.KVCache(tk, tv, pt)
+    st = _status()
+    f = lambda a: torch.from_numpy(a).cuda()
+    dreams.kv_compact(kv, f(L), f(acc), f(path), status=st)
+    assert int(st.item()) == 0
+    assert np.array_equal(tk.view(torch.int16).cpu().numpy().view(np.uint16), ko)
+    assert np.array_equal(tv.view(torch.int16).cpu().numpy().view(np.uint16), vo)
+
+
+def test_kv_compact_bad_path_untouched(dreams):
+    B, cap, Hkv, D = 3, 64, 1, 64
+    k = torch.randn((B, cap, Hkv, D)).to(torch.bfloat16).cuda()
+    k0 = k.clone()
+    kv = dreams.KVCache(k, k.clone())
+    path = torch.tensor([[1, 2, 3], [0, 2, 2], [0, 1, 60]], dtype=torch.int32, device="cuda")
+    st = _status()
+    dreams.kv_compact(kv, torch.tensor([0, 0, 10], dtype=torch.int32, device="cuda"),
+                      torch.tensor([3, 3, 3], dtype=torch.int32, device="cuda"), path, status=st)
+    s = int(st.item())
+    assert s & dreams.DATA_BAD_PATH and s & dreams.DATA_BAD_KV_LEN
+    assert torch.equal(k, k0)
+
+
+# ------------------------------------------------------------------ fused step
+@pytest.mark.parametrize("name", CONFIGS)
+def test_verify_step_matches_oracle(dreams, name):
+    w = W.make(name)
+    g = to_gpu(w)
+    max_path = w.max_path
+    am_out = torch.full((w.B, w.T_max), -7, dtype=torch.int32, device="cuda")
+    st = _status()
+    r = dreams.verify_step(g["logits"], g["tree"], g["kv"], max_path, argmax_out=am_out, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    am_ref = logits_rows_oracle(w)
+    am_gpu = am_out.cpu().numpy()
+    for b in range(w.B):
+        t = int(w.tree_len[b])
+        np.testing.assert_array_equal(am_gpu[b, :t], am_ref[b, :t])
+        assert (am_gpu[b, t:] == -7).all()
+    ref = oracle.accept_path(am_ref, w.parent.numpy(), w.tokens.numpy(), w.tree_len.numpy(),
+                             w.kv_len.numpy(), max_path)
+    for key in ("accept_len", "path", "out_tokens", "new_kv_len"):
+        np.testing.assert_array_equal(r[key].cpu().numpy(), ref[key], err_msg=key)
+    # planted structure: mean acceptance is well above 1
+    assert ref["accept_len"].mean() > 1.5
+    ko, vo, ost = oracle.kv_compact(W.bits(w.k), W.bits(w.v), layout(w), w.kv_len.numpy(), ref["accept_len"],
+                                    ref["path"])
+    assert ost == 0
+    assert np.array_equal(W.bits(g["k"].cpu()), ko)
+    assert np.array_equal(W.bits(g["v"].cpu()), vo)
+
+
+def test_verify_step_bad_sequences(dreams):
+    """Bad data in one sequence is reported and leaves the others intact."""
+    w = W.make("batched", with_attn=True)
+    am_ref = logits_rows_oracle(w)
+    ref = oracle.accept_path(am_ref, w.parent.numpy(), w.tokens.numpy(), w.tree_len.numpy(), w.kv_len.numpy(),
+                             w.max_path)
+    pb = [b for b in range(9, w.B) if ref["accept_len"][b] >= 2][0]  # has moves to make
+    par = w.parent.clone()
+    par[2, 5] = 7            # parent not below the node
+    tl = w.tree_len.clone()
+    tl[4] = 0                # empty tree
+    kl = w.kv_len.clone()
+    kl[6] = w.capacity       # no room for the tree
+    pt = w.page_table.clone()
+    lo, hi = int(w.kv_len[pb]) // 64, (int(w.kv_len[pb]) + int(w.tree_len[pb]) - 1) // 64
+    pt[pb, lo:hi + 1] = w.num_pages + 3  # bad pages under the tree slots
+    w2 = W.Workload(**{**w.__dict__, "parent": par, "tree_len": tl, "kv_len": kl, "page_table": pt})
+    g = to_gpu(w2)
+    st = _status()
+    r = dreams.verify_step(g["logits"], g["tree"], g["kv"], w.max_path, status=st)
+    s = int(st.item())
+    assert s & dreams.DATA_BAD_PARENT and s & dreams.DATA_BAD_TREE_LEN and s & dreams.DATA_BAD_KV_LEN
+    assert s & dreams.DATA_BAD_PAGE
+    acc = r["accept_len"].cpu().numpy()
+    assert acc[2] == 0 and acc[4] == 0 and acc[6] == 0
+    good = [b for b in range(w.B) if b not in (2, 4, 6, pb)]
+    np.testing.assert_array_equal(acc[good], ref["accept_len"][good])
+
+
+def test_status_word_clean_on_valid_input(dreams):
+    w = W.make("tiny")
+    g = to_gpu(w)
+    st = _status()
+    dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, status=st)
+    dreams.verify_step(g["logits"], g["tree"], g["kv"], w.max_path, status=st)
+    assert int(st.item()) == 0
