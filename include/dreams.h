@@ -25,11 +25,12 @@
  * ---------------------------------------
  *  - All data pointers are DEVICE pointers owned by the caller; the library
  *    allocates no memory. Scratch comes from a caller-supplied workspace
- *    whose size the matching *_workspace_size function returns. A workspace
- *    must be zero-filled once when it is allocated; every call leaves it
- *    zero-filled again (its counters reset themselves), so it can be reused
- *    by later calls on the same stream. Calls that overlap in time must not
- *    share a workspace.
+ *    (16-byte aligned) whose size the matching *_workspace_size function
+ *    returns. The attention workspace holds no state between calls. The
+ *    argmax and verify-step workspaces hold counters that reset themselves:
+ *    zero-fill such a workspace once when it is allocated, and every call
+ *    leaves it zero-filled again, whatever its shape arguments. Calls that
+ *    overlap in time must not share a workspace.
  *  - Every call is asynchronous on the given stream (NULL = the legacy
  *    default stream) and runs on the current CUDA device.
  *  - Host-side checks (null pointers, sizes, alignment, supported shapes)
@@ -79,6 +80,7 @@ typedef enum dreams_dtype { DREAMS_F32 = 0, DREAMS_BF16 = 1 } dreams_dtype_t;
 #define DREAMS_DATA_BAD_KV_LEN 0x4   /* kv_len < 0 or kv_len + tree_len > capacity */
 #define DREAMS_DATA_BAD_PAGE 0x8     /* page-table entry outside [0, num_pages) */
 #define DREAMS_DATA_BAD_PATH 0x10    /* path[0] != 0 or not strictly increasing */
+#define DREAMS_DATA_TIMEOUT 0x20     /* a kernel gave up waiting on its own pipeline (2 s) */
 
 /*
  * One attention layer's K and V cache (bf16), or n_layers of them.

@@ -487,6 +487,7 @@ struct StepParams {
   KVParams kv;
   int32_t max_path;
   int32_t *pred;  // [B, T_max] predictions (caller's argmax_out or workspace)
+  bool pred_in_ws;
   int32_t *seq_cnt;
   int32_t *accept_len, *path, *out_tokens, *new_kv_len;
   int32_t *status;
@@ -546,6 +547,10 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_step_kernel(const StepPar
     }
     write_walk(b, w.n, L, p.tr.tokens + rb, p.pred + rb, s_path, p.max_path, p.accept_len, p.path, p.out_tokens,
                p.new_kv_len);
+    if (p.pred_in_ws) {  // leave the workspace zero-filled
+      __syncwarp();
+      for (int x = threadIdx.x; x < tl; x += 32) p.pred[rb + x] = 0;
+    }
     bool ok = w.n > 0;
     if (ok) ok = move_offsets(p.kv, b, L, w.n, s_path, s_src, s_dst, p.status);
     if (threadIdx.x == 0) s_go = ok ? w.n : 0;
@@ -711,6 +716,7 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   int32_t *ws_pred = reinterpret_cast<int32_t *>(ws + argmax_ws(rows));
   p.seq_cnt = reinterpret_cast<int32_t *>(ws + argmax_ws(rows) + align_up(size_t(rows) * 4, 256));
   p.pred = argmax_out != nullptr ? argmax_out : ws_pred;
+  p.pred_in_ws = argmax_out == nullptr;
   p.max_path = max_path;
   p.accept_len = accept_len;
   p.path = path;
