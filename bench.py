@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
+    ap.add_argument("--load-seconds", type=float, default=1.0,
+                    help="untimed steps run while the clock sampler starts (0 under a profiler)")
     return ap.parse_args()
 
 
@@ -69,6 +71,22 @@ def argmax_bytes(w: W.Workload) -> int:
 def attn_flops(w: W.Workload) -> int:
     return int(sum(4 * int(w.tree_len[b]) * w.Hq * (int(w.kv_len[b]) + int(w.tree_len[b])) * w.D
                    for b in range(w.B)))
+
+
+def measured_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    kernel source has not changed since it was captured (else None)."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)[kernel]
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+    except (OSError, KeyError, ValueError):
+        return None
+    if sha != rec["source_sha256"] or rec["workload"] != workload:
+        return None
+    return int(rec["dram_bytes_per_launch"])
 
 
 def peaks():
@@ -192,7 +210,7 @@ def run_dreams(args, rank, world, local):
     clocks = ClockSampler(local)
     clocks.start()
     t_load = time.time()  # keep the GPU busy ~1 s so the sampler sees the clocks under this load
-    while time.time() - t_load < 1.0:
+    while time.time() - t_load < args.load_seconds:
         for i in range(20):
             step(copies[i % 2])
         torch.cuda.synchronize(dev)
@@ -260,7 +278,7 @@ def run_dreams(args, rank, world, local):
         "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
         "frac_of_nominal_8000": round(achieved / NOMINAL_HBM_GBS, 4),
         "algorithmic_bytes": ab, "avg_launch_us": round(attn_avg_ms * 1000, 2),
-        "traffic": None,
+        "traffic": measured_traffic("tree_attn_tc_kernel", w.spec.name),
     }
     tail_gbs = gb / (tail_avg_ms * 1e-3) / 1e9
     kernels = {
