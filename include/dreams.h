@@ -69,7 +69,8 @@ typedef enum dreams_status {
   DREAMS_ERR_INVALID_ARG = 1, /* null pointer, bad size, misaligned pointer */
   DREAMS_ERR_UNSUPPORTED = 2, /* valid but unsupported shape or dtype */
   DREAMS_ERR_WORKSPACE = 3,   /* workspace missing or too small */
-  DREAMS_ERR_CUDA = 4         /* a CUDA call failed; see dreams_last_cuda_error */
+  DREAMS_ERR_CUDA = 4,        /* a CUDA call failed; see dreams_last_cuda_error */
+  DREAMS_ERR_SCRATCH_LIMIT = 5 /* larger than a no-allocation entry point's fixed scratch */
 } dreams_status_t;
 
 typedef enum dreams_dtype { DREAMS_F32 = 0, DREAMS_BF16 = 1 } dreams_dtype_t;
@@ -200,6 +201,35 @@ dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int
                                    int32_t *accept_len, int32_t *path, int32_t *out_tokens,
                                    int32_t *new_kv_len, void *workspace, size_t workspace_bytes,
                                    int32_t *status_word, dreams_stream_t stream);
+
+/*
+ * Row-wise argmax for callers that cannot allocate device memory. The paper
+ * has no counterpart to this call; it exists for integration. Some callers
+ * cannot allocate, or cannot hand out a workspace, when the argmax runs: a
+ * plugin inside an inference engine that owns and plans all device memory and
+ * gives the plugin no way to ask for more at run time; a serving process that
+ * reserves its whole memory budget at start-up and treats any later allocation
+ * as an error; a latency-critical loop in which an allocation's implicit
+ * synchronisation would stall other streams.
+ *
+ * Same result and arguments as dreams_vocab_argmax, without the workspace: the
+ * scratch is a fixed device array inside this library (12 bytes per row for
+ * DREAMS_NOALLOC_ARGMAX_MAX_ROWS rows, about 192 KiB), which every GPU that
+ * loads the library holds until the process exits. The call allocates and
+ * frees nothing; it clears the part of the scratch it uses with
+ * cudaMemsetAsync on the given stream, then launches the argmax kernel.
+ *  - rows > DREAMS_NOALLOC_ARGMAX_MAX_ROWS returns DREAMS_ERR_SCRATCH_LIMIT
+ *    and launches nothing.
+ *  - The first call on each device looks up the scratch's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - All calls share the one scratch array: calls that overlap on the GPU
+ *    (different streams, or different host threads) race and may return
+ *    wrong indices. Serialise them, e.g. on one stream.
+ */
+#define DREAMS_NOALLOC_ARGMAX_MAX_ROWS 16384
+dreams_status_t dreams_vocab_argmax_noalloc(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
+                                            int64_t row_stride, int32_t *out_idx, dreams_stream_t stream);
 
 const char *dreams_status_string(dreams_status_t status);
 int32_t dreams_version(void);

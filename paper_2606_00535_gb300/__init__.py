@@ -30,7 +30,8 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libdreams.so")
 HEADER = os.path.join(os.path.dirname(_HERE), "include", "dreams.h")
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SCRATCH_LIMIT = 0, 1, 2, 3, 4, 5
+NOALLOC_ARGMAX_MAX_ROWS = 16384
 F32, BF16 = 0, 1
 DATA_BAD_PARENT, DATA_BAD_TREE_LEN, DATA_BAD_KV_LEN, DATA_BAD_PAGE, DATA_BAD_PATH = 1, 2, 4, 8, 16
 
@@ -83,6 +84,7 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step_workspace_size": (sz, [ptr, i64]),
                     "dreams_verify_step": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, p, p, p, p,
                                                           p, p, sz, p, p]),
+                    "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
                     "dreams_status_string": (ctypes.c_char_p, [ctypes.c_int]),
                     "dreams_version": (i32, []),
                     "dreams_last_cuda_error": (i32, []),
@@ -262,6 +264,25 @@ def vocab_argmax(logits: torch.Tensor, out: Optional[torch.Tensor] = None,
         _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), _ptr(out),
         _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
     _check("dreams_vocab_argmax", st)
+    return out
+
+
+def vocab_argmax_noalloc(logits: torch.Tensor, out: torch.Tensor, stream=None) -> torch.Tensor:
+    """Row-wise argmax into a caller-provided ``out`` without any device
+    allocation, for callers that must not allocate while it runs (see
+    ``dreams_vocab_argmax_noalloc`` in include/dreams.h): the library's fixed
+    scratch serves at most NOALLOC_ARGMAX_MAX_ROWS rows, and calls that overlap
+    on the GPU race."""
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    V = int(logits.shape[-1])
+    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
+    if x.stride(-1) != 1:
+        raise ValueError("logits rows must be contiguous")
+    _need(out, "out", torch.int32, logits.device)
+    st = _lib().dreams_vocab_argmax_noalloc(_ptr(x), F32 if x.dtype == torch.float32 else BF16, int(x.shape[0]), V,
+                                            int(x.stride(0)), _ptr(out), _stream(stream))
+    _check("dreams_vocab_argmax_noalloc", st)
     return out
 
 

@@ -35,6 +35,7 @@ extern "C" const char *dreams_status_string(dreams_status_t status) {
     case DREAMS_ERR_UNSUPPORTED: return "unsupported shape or dtype";
     case DREAMS_ERR_WORKSPACE: return "workspace missing or too small";
     case DREAMS_ERR_CUDA: return "CUDA error";
+    case DREAMS_ERR_SCRATCH_LIMIT: return "problem larger than the fixed scratch of a no-allocation entry point";
   }
   return "unknown status";
 }

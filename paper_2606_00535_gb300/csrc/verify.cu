@@ -26,6 +26,7 @@
 #include <limits.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -727,5 +728,85 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (dtype == DREAMS_F32) verify_step_kernel<float><<<grid, TAIL_THREADS, 0, s>>>(p);
   else verify_step_kernel<__nv_bfloat16><<<grid, TAIL_THREADS, 0, s>>>(p);
+  return check_launch();
+}
+
+// ------------------------------------------------------------------ no-allocation argmax
+// Scratch of dreams_vocab_argmax_noalloc: a fixed file-scope device array that
+// every GPU loading this library holds until the process exits. Host code
+// must not hand g_noalloc_scratch to a kernel directly (in host code that
+// name is a host-side stand-in, not a device address): its device address is
+// looked up with cudaGetSymbolAddress once per device.
+namespace {
+constexpr int64_t NOALLOC_ROWS = DREAMS_NOALLOC_ARGMAX_MAX_ROWS;
+constexpr size_t NOALLOC_SLOT_BYTES = size_t(NOALLOC_ROWS) * 8;  // one (key, index) word per row
+constexpr size_t NOALLOC_BYTES = NOALLOC_SLOT_BYTES + size_t(NOALLOC_ROWS) * 4;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
+
+std::mutex g_noalloc_mutex;
+void *g_noalloc_ptr[64] = {nullptr};
+
+// Device address of the scratch on the current device (looked up on the first
+// call per device, which must happen outside any stream capture).
+dreams_status_t noalloc_scratch(void **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= 64) return DREAMS_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void *ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess || ptr == nullptr) {
+      set_last_cuda_error(e);
+      return DREAMS_ERR_CUDA;
+    }
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return DREAMS_OK;
+}
+}  // namespace
+
+extern "C" dreams_status_t dreams_vocab_argmax_noalloc(const void *logits, dreams_dtype_t dtype, int64_t rows,
+                                                       int64_t V, int64_t row_stride, int32_t *out_idx,
+                                                       dreams_stream_t stream) {
+  if (logits == nullptr || out_idx == nullptr || rows < 1 || V < 1 || V > INT_MAX || row_stride < V)
+    return DREAMS_ERR_INVALID_ARG;
+  if (dtype != DREAMS_F32 && dtype != DREAMS_BF16) return DREAMS_ERR_UNSUPPORTED;
+  if (rows > NOALLOC_ROWS) return DREAMS_ERR_SCRATCH_LIMIT;
+  const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
+  if (reinterpret_cast<uintptr_t>(logits) % esz) return DREAMS_ERR_INVALID_ARG;
+  const ArgmaxPlan pl = plan_argmax(rows, V);
+  if (rows * pl.nchunk > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  void *scratch = nullptr;
+  dreams_status_t st = noalloc_scratch(&scratch);
+  if (st != DREAMS_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  ArgmaxParams p{};
+  p.logits = logits;
+  p.V = V;
+  p.row_stride = row_stride;
+  p.chunk = pl.chunk;
+  p.nchunk = pl.nchunk;
+  p.vec_ok = aligned16(logits) && (row_stride * int64_t(esz)) % 16 == 0;
+  p.out = out_idx;
+  p.slot = static_cast<unsigned long long *>(scratch);
+  p.cnt = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(scratch) + NOALLOC_SLOT_BYTES);
+  if (pl.nchunk > 1) {
+    // the row slots and counters must start at zero
+    cudaError_t e = cudaMemsetAsync(p.slot, 0, size_t(rows) * 8, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(p.cnt, 0, size_t(rows) * 4, s);
+    if (e != cudaSuccess) {
+      set_last_cuda_error(e);
+      return DREAMS_ERR_CUDA;
+    }
+  }
+  const dim3 grid(unsigned(rows * pl.nchunk));
+  if (dtype == DREAMS_F32) vocab_argmax_kernel<float><<<grid, ARGMAX_THREADS, 0, s>>>(p);
+  else vocab_argmax_kernel<__nv_bfloat16><<<grid, ARGMAX_THREADS, 0, s>>>(p);
   return check_launch();
 }

@@ -23,7 +23,7 @@ def lib():
 
 def test_exports_every_declared_function(lib):
     names = dreams.declared_functions()
-    assert len(names) == 11
+    assert len(names) >= 11
     for n in names:
         assert hasattr(lib, n), n
     out = subprocess.run(["nm", "-D", "--defined-only", dreams.LIB_PATH], capture_output=True, text=True).stdout
