@@ -129,8 +129,9 @@ typedef struct dreams_tree {
  * q, out: bf16 [B, T_max, Hq, D] (16-byte aligned). lse: f32 [B, T_max, Hq]
  * or NULL. Rows t >= tree_len[b] of out and lse are left untouched, and so are
  * all rows of a sequence with bad data. layer selects the cache
- * (0 <= layer < kv->n_layers). Accumulation is fp32; the output is rounded to
- * bf16 once.
+ * (0 <= layer < kv->n_layers). scale must be finite and > 0. Accumulation is
+ * fp32 (the probabilities enter the PV product as bf16); the output is
+ * rounded to bf16 once.
  */
 size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
                                               int32_t Hq);
