@@ -48,9 +48,10 @@ def test_binding_fails_loudly_without_library(tmp_path):
 def test_workspace_sizes(lib):
     k = torch.empty(0, dtype=torch.bfloat16)
     kvc = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
-    tr = dreams._Tree(16, 16, 16, 16, 16, 64)
-    n = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32)
+    one = dreams._Tree(16, 16, 16, 16, 1, 64)     # one sequence: the KV range is split over CTAs
+    n = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 32)
     assert n > 0 and n % 256 == 0
+    tr = dreams._Tree(16, 16, 16, 16, 16, 64)
     bad = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
     assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(bad), ctypes.byref(tr), 30) == 0
     assert lib.dreams_vocab_argmax_workspace_size(768, 128256) >= 0
