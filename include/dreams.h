@@ -126,6 +126,7 @@ typedef struct dreams_tree {
  *     keys  J = { slots 0 .. L_b - 1 } U { slot L_b + a : a = t or an ancestor of t }
  *     out[b, t, h, :] = sum_{j in J} softmax_j(scale * <q, K[b, j, g]>) V[b, j, g, :]
  *     lse[b, t, h]    = log sum_{j in J} exp(scale * <q, K[b, j, g]>)
+ * Hq must be a multiple of kv->Hkv with at most 128 query heads per KV head.
  * q, out: bf16 [B, T_max, Hq, D] (16-byte aligned). lse: f32 [B, T_max, Hq]
  * or NULL. Rows t >= tree_len[b] of out and lse are left untouched, and so are
  * all rows of a sequence with bad data. layer selects the cache

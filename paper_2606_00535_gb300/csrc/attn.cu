@@ -7,17 +7,25 @@
 // and query head h, softmax attention over the prefix slots 0..L-1 and the
 // slots L + a of t and its ancestors a, with KV head g = h / G.
 //
-// Work decomposition: one CTA per (KV split, KV head g, sequence b, block of
-// 128 query rows), one CTA per SM. The query rows of a CTA are the (tree node
-// t, head h - gG) pairs, row = t * G + (h - gG), so one pass over a K/V tile
-// serves every query head of the GQA group and every tree node.
+// Work decomposition: one CTA per work item (sequence b, KV split, KV head g,
+// row block rb), one CTA per SM. A row block holds TB = 128 / G tree nodes
+// times the G query heads of the group, row = (t - rb*TB) * G + (h - gG), so
+// one pass over a K/V tile serves every query head of the GQA group and every
+// tree node of the block. With more than one sequence, a one-CTA kernel first
+// orders the (sequence, split) pairs longest first, so that the hardware,
+// which hands out CTAs in index order as SMs free up, schedules the items
+// longest-processing-time first.
 //
 // Roles (320 threads):
-//   warp 8, one thread  TMA producer: 128-token K tiles into a 2-stage ring and
-//                       V tiles into a 3-stage ring (4-D boxes of 64 slots x
-//                       64 head columns, 128-byte swizzle). A K stage is
-//                       released as soon as its QK^T has run, a V stage after
-//                       its PV.
+//   warp 8, one thread  TMA producer: the Q block first (one 5-D box per
+//                       64-column region), then 128-token K tiles into a
+//                       3-stage ring and V tiles into a 3-stage ring (4-D
+//                       boxes of 64 slots x 64 head columns, 128-byte
+//                       swizzle). It polls both rings without blocking and
+//                       keeps V a tile behind K (QK^T of tile j + 1 runs
+//                       before PV of tile j); page-table entries are loaded
+//                       one tile ahead. A K stage is released as soon as its QK^T
+//                       has run, a V stage after its PV.
 //   warp 9, one thread  MMA issuer: S = Q K^T (M128 N128, K-major operands) into
 //                       TMEM, O += P V (M128 N=D, P read from TMEM, V as an
 //                       MN-major operand). Tile j goes to warpgroup j % 2, and
@@ -35,12 +43,15 @@
 //                       exceeds it by 2^8 (and only then rescales its O), and
 //                       writes P as bf16 over S. Warps whose rows are all
 //                       padding sit out.
-// At the end the two warpgroups combine their (m, l, O) by log-sum-exp and
-// write the output, or the split partials that a second kernel (chained by
-// programmatic dependent launch) merges. Every mbarrier wait is bounded (2 s);
-// on a timeout the CTA flags DREAMS_DATA_TIMEOUT, drains its copies and MMAs,
-// frees its TMEM and exits. The workspace holds no state between calls.
+// At the end the two warpgroups combine their (m, l, O) by log-sum-exp into a
+// swizzled staging copy in the idle shared-memory rings, and all 256 threads
+// write it out in row order (16-byte coalesced stores): the output, or the
+// split partials that a merge kernel (chained by programmatic dependent
+// launch) combines. Every mbarrier wait is bounded (2 s); on a timeout the CTA
+// flags DREAMS_DATA_TIMEOUT, drains its copies and MMAs, frees its TMEM and
+// exits. The workspace holds no state between calls.
 #include <cuda.h>
+#include <limits.h>
 #include <math.h>
 #include <string.h>
 
@@ -57,12 +68,17 @@ constexpr float LN2 = 0.6931471805599453f;
 
 constexpr int KT = 128;        // KV tokens per tile (UMMA N of QK^T)
 constexpr int ROWS = 128;      // query rows per CTA (UMMA M)
-constexpr int NK = 2;          // K ring stages
+constexpr int NK = 3;          // K ring stages
 constexpr int NV = 3;          // V ring stages
+constexpr int CRD = 8;         // producer's ring of tile coordinates (V trails K by < CRD tiles)
 constexpr int THREADS = 320;   // 8 softmax warps, TMA warp, MMA warp
 constexpr int TMA_WARP = 8, MMA_WARP = 9;
 constexpr float RESCALE = 8.f; // log2 headroom of the reference maximum
 constexpr uint32_t TMEM_COLS = 512;
+constexpr int MAX_SPLITS = 32; // KV splits per sequence (one merge lane each)
+constexpr int ORDER_THREADS = 1024;
+constexpr int ORDER_KEYS = 4096;  // item sizes (tiles) above this share the top bucket
+constexpr int PAST_TABLE = INT_MIN;  // page-table slot past the table: reads as zeros
 
 struct AttnParams {
   const __nv_bfloat16 *q;
@@ -76,16 +92,19 @@ struct AttnParams {
   const int32_t *tree_len;
   const int32_t *kv_len;
   int32_t B, T_max, Hq, Hkv, G;
-  int32_t nrb;     // 128-row blocks per (b, g)
-  int32_t nsplit;  // KV splits in the grid
+  int32_t TB;      // tree nodes per row block (ROWS / G)
+  int32_t nrb;     // row blocks per (b, g)
+  int32_t nsplit;  // KV splits per sequence in the grid
   int32_t chunk;   // KV tokens per split, a multiple of KT
   float scale_log2;
-  float *ws_o;    // [B][Hkv][nrb][nsplit][ROWS][D] unnormalised partial O
-  float2 *ws_ml;  // [B][Hkv][nrb][nsplit][ROWS] (max in log2 units, sum)
+  float *ws_o;     // [B][Hkv][nrb][nsplit][ROWS][D] unnormalised partial O
+  float2 *ws_ml;   // [B][Hkv][nrb][nsplit][ROWS] (max in log2 units, sum)
+  int32_t *order;  // [B * nsplit] pair index b * nsplit + split, longest first; nullptr: natural order
   int32_t *status;
 };
 
 struct TcParams {
+  CUtensorMap tmap_q;
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;
   AttnParams a;
@@ -94,6 +113,72 @@ struct TcParams {
 
 __device__ __forceinline__ void named_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// KV tiles of split s of sequence b (0 for an empty split or bad lengths).
+__device__ __forceinline__ int split_tiles(const AttnParams &p, int b, int s) {
+  const int T = __ldg(p.tree_len + b);
+  const int L = __ldg(p.kv_len + b);
+  if (T < 1 || T > p.T_max || L < 0 || L > p.capacity - T) return 0;
+  const int tiles = (L + T + KT - 1) / KT;
+  const int ct = p.chunk / KT;
+  return ::max(0, ::min(ct, tiles - s * ct));
+}
+
+// Orders the (sequence, split) pairs by their number of KV tiles, largest
+// first (a counting sort; pairs of equal size may come in any order, which
+// changes only which SM computes them, not the result).
+__global__ void __launch_bounds__(ORDER_THREADS) tree_attn_order_kernel(const AttnParams p) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  __shared__ int bucket[ORDER_KEYS];
+  __shared__ int warp_sum[ORDER_THREADS / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int P = p.B * p.nsplit;
+  for (int k = tid; k < ORDER_KEYS; k += ORDER_THREADS) bucket[k] = 0;
+  __syncthreads();
+  for (int e = tid; e < P; e += ORDER_THREADS) {
+    const int b = e / p.nsplit;
+    atomicAdd(&bucket[::min(split_tiles(p, b, e - b * p.nsplit), ORDER_KEYS - 1)], 1);
+  }
+  __syncthreads();
+  // start of key k = number of pairs with a larger key; thread t owns keys
+  // ORDER_KEYS-1-4t down to ORDER_KEYS-4-4t
+  int v[4], sum = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    v[i] = bucket[ORDER_KEYS - 1 - 4 * tid - i];
+    sum += v[i];
+  }
+  int x = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = warp_sum[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    warp_sum[lane] = w;
+  }
+  __syncthreads();
+  int run = x - sum + (warp > 0 ? warp_sum[warp - 1] : 0);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    bucket[ORDER_KEYS - 1 - 4 * tid - i] = run;
+    run += v[i];
+  }
+  __syncthreads();
+  for (int e = tid; e < P; e += ORDER_THREADS) {
+    const int b = e / p.nsplit;
+    const int pos = atomicAdd(&bucket[::min(split_tiles(p, b, e - b * p.nsplit), ORDER_KEYS - 1)], 1);
+    p.order[pos] = e;
+  }
 }
 
 template <int D>
@@ -110,16 +195,24 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t bar_kf[NK], bar_ke[NK], bar_vf[NV], bar_ve[NV];
-  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_drain;
+  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_q, bar_drain;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_zero, s_flag;
   __shared__ unsigned long long s_anc[64];
   __shared__ int s_jump[64];
-  __shared__ float2 s_ml[2][ROWS];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int rb = blockIdx.x % p.nrb, split = blockIdx.x / p.nrb;
-  const int g = blockIdx.y, b = blockIdx.z;
+  const int per_pair = p.Hkv * p.nrb;
+  const int pair_pos = blockIdx.x / per_pair;
+  const int gr = blockIdx.x - pair_pos * per_pair;
+  const int g = gr / p.nrb, rb = gr - g * p.nrb;
+  int pair = pair_pos;
+  if (p.order != nullptr) {
+    // the order comes from the preceding kernel (programmatic dependent launch)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    pair = __ldcg(p.order + pair_pos);
+  }
+  const int b = pair / p.nsplit, split = pair - b * p.nsplit;
   const bool reporter = (rb == 0 && split == 0 && g == 0);
   const int T = __ldg(p.tree_len + b);
   const int L = __ldg(p.kv_len + b);
@@ -133,10 +226,11 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   }
   const int total = L + T;
   const int nsplit_b = (total + p.chunk - 1) / p.chunk;
-  const int rows_b = T * p.G;
-  if (split >= nsplit_b || rb * ROWS >= rows_b) return;
+  const int t0 = rb * p.TB;  // first tree node of the row block
+  if (split >= nsplit_b || t0 >= T) return;
+  const int rows_blk = ::min(p.TB, T - t0) * p.G;  // real query rows of this CTA
   // softmax warps whose 32 rows hold at least one real query row
-  const int n_act = min(4, (rows_b - rb * ROWS + 31) / 32);
+  const int n_act = ::min(4, (rows_blk + 31) / 32);
 
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t q_s = smem_base;
@@ -145,7 +239,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const uint32_t kf0 = smem_u32(&bar_kf[0]), ke0 = smem_u32(&bar_ke[0]);
   const uint32_t vf0 = smem_u32(&bar_vf[0]), ve0 = smem_u32(&bar_ve[0]);
   const uint32_t bs0 = smem_u32(&bar_s[0]), bp0 = smem_u32(&bar_p[0]);
-  const uint32_t bdrain = smem_u32(&bar_drain);
+  const uint32_t bq = smem_u32(&bar_q), bdrain = smem_u32(&bar_drain);
 
   if (tid == TMA_WARP * 32) {
     for (int i = 0; i < NK; ++i) {
@@ -160,6 +254,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       tc::mbar_init(bs0 + 8 * i, 1);
       tc::mbar_init(bp0 + 8 * i, 32 * n_act);
     }
+    tc::mbar_init(bq, 1);
     tc::mbar_init(bdrain, 1);
     s_abort = 0;
     s_zero = 0;
@@ -175,7 +270,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const uint32_t tmem = s_tmem;
 
   const int c0 = split * p.chunk;
-  const int c1 = min(c0 + p.chunk, total);
+  const int c1 = ::min(c0 + p.chunk, total);
   const int ntiles = (c1 - c0 + KT - 1) / KT;
   volatile int *abort_flag = &s_abort;
   // abort codes: 1 = a wait timed out, 2 = malformed tree (nothing to compute)
@@ -186,13 +281,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     }
   };
 
-  // While the producer starts streaming K/V, the MMA warp checks the tree and
-  // builds the ancestor masks and the softmax warps stage Q; named barrier 2
-  // (MMA warp + softmax warps) publishes both.
+  // While the producer streams Q, K and V, the MMA warp checks the tree and
+  // builds the ancestor masks; named barrier 2 (MMA warp + softmax warps)
+  // publishes them.
   const int wg = warp >> 2;                  // softmax warpgroup (warps 0-7)
   const int row = 32 * (warp & 3) + lane;    // TMEM lane = query row
-  const int grow = rb * ROWS + row;
-  const int t_row = grow / p.G;
+  const bool real_row = row < rows_blk;
+  const int t_row = t0 + row / p.G;
   if (warp == MMA_WARP) {
     int par[2], bad = 0;
 #pragma unroll
@@ -239,78 +334,99 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     }
     named_sync(2, 288);
   } else if (warp < 8) {
-    // Q rows -> shared memory (128-byte-swizzled K-major layout); the two
-    // warpgroups fill the two halves of each row
-    const bool ok = grow < rows_b;
-    const int hg = grow - t_row * p.G;
-    const uint4 *src = reinterpret_cast<const uint4 *>(
-        p.q + ((int64_t(b) * p.T_max + (ok ? t_row : 0)) * p.Hq + g * p.G + hg) * D);
-#pragma unroll
-    for (int cc = 0; cc < D / 16; ++cc) {
-      const int c = wg * (D / 16) + cc;
-      const uint4 v = ok ? __ldg(src + c) : make_uint4(0u, 0u, 0u, 0u);
-      const uint32_t dst = q_s + (c >> 3) * Q_REGION + row * 128 + (((c & 7) ^ (row & 7)) << 4);
-      asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                   : "memory");
-    }
-    tc::fence_proxy_async_smem();
     named_sync(2, 288);
   }
   const bool tree_ok = (warp == TMA_WARP) || !s_flag;
 
+  float m_ref = -INFINITY, l = 0.f;  // this thread's row state (softmax warps)
+  bool sm_ok = false;                // the softmax loop ran to completion
+
   if (warp == TMA_WARP) {
     // ---------------- TMA producer
     if (lane == 0) {
+      tc::prefetch_tmap(&P.tmap_q);
       tc::prefetch_tmap(&P.tmap_k);
       tc::prefetch_tmap(&P.tmap_v);
-      int nk = 0, nv = 0;  // tiles issued into each ring
-      for (int j = 0; j < ntiles; ++j) {
-        if (*abort_flag) break;
-        const int s0 = c0 + j * KT;
-        int c2[2], c3[2];  // coordinates of the two 64-slot halves of the tile
+      // the Q rows of the block: G heads x TB nodes per 64-column region
+      // (nodes past T_max read as zeros; the transaction counts the full box)
+      tc::mbar_arrive_expect_tx(bq, uint32_t(NR * p.G * p.TB * 128));
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          if (P.paged) {
-            int pg = __ldg(p.page_table + int64_t(b) * p.pages_per_seq + ((s0 >> 6) + h));
-            if ((s0 >> 6) + h >= p.pages_per_seq) pg = p.num_pages;  // past the table: zeros
-            else if (pg < 0 || pg >= p.num_pages) {
-              if (s0 + 64 * h < c1) flag(p.status, DREAMS_DATA_BAD_PAGE);
-              pg = p.num_pages;  // outside the tensor map: the copy fills zeros
-            }
-            c2[h] = 0;
-            c3[h] = pg;
-          } else {
-            c2[h] = s0 + 64 * h;
-            c3[h] = b;
+      for (int r = 0; r < NR; ++r) tc::tma_load_5d(q_s + r * Q_REGION, &P.tmap_q, bq, r * 64, 0, g, t0, b);
+      // raw page-table entries of the two 64-slot halves of tile j
+      const int32_t *prow = P.paged ? p.page_table + int64_t(b) * p.pages_per_seq : nullptr;
+      auto fetch = [&](int j, int &e0, int &e1) {
+        if (P.paged && j < ntiles) {
+          const int pi = (c0 + j * KT) >> 6;
+          e0 = pi < p.pages_per_seq ? __ldg(prow + pi) : PAST_TABLE;
+          e1 = pi + 1 < p.pages_per_seq ? __ldg(prow + pi + 1) : PAST_TABLE;
+        }
+      };
+      // tensor-map coordinate (dim 3) of half h of tile j
+      auto page_coord = [&](int j, int h, int e) {
+        if (!P.paged) return b;
+        if (e == PAST_TABLE) return p.num_pages;  // past the table: the copy fills zeros
+        if (e < 0 || e >= p.num_pages) {
+          if (c0 + j * KT + 64 * h < c1) flag(p.status, DREAMS_DATA_BAD_PAGE);
+          return p.num_pages;  // outside the tensor map: the copy fills zeros
+        }
+        return e;
+      };
+      int ring[CRD][2];
+      int pn0 = 0, pn1 = 0;
+      fetch(0, pn0, pn1);
+      int nk = 0, nv = 0;  // tiles issued into each ring
+      uint32_t idle = 0;
+      uint64_t t_idle = 0;
+      while (nv < ntiles && !*abort_flag) {
+        bool progress = false;
+        if (nk < ntiles && nk - nv < CRD &&
+            (nk < NK || tc::mbar_test_wait(ke0 + 8 * (nk % NK), ((nk / NK) - 1) & 1))) {
+          const int c3a = page_coord(nk, 0, pn0), c3b = page_coord(nk, 1, pn1);
+          ring[nk % CRD][0] = c3a;
+          ring[nk % CRD][1] = c3b;
+          fetch(nk + 1, pn0, pn1);
+          const int ks = nk % NK, s0 = c0 + nk * KT;
+          tc::mbar_arrive_expect_tx(kf0 + 8 * ks, KV_TILE);
+#pragma unroll
+          for (int r = 0; r < NR; ++r) {
+            tc::tma_load_4d(k_s(ks) + r * KV_REGION, &P.tmap_k, kf0 + 8 * ks, r * 64, g, P.paged ? 0 : s0, c3a);
+            tc::tma_load_4d(k_s(ks) + r * KV_REGION + 8192, &P.tmap_k, kf0 + 8 * ks, r * 64, g,
+                            P.paged ? 0 : s0 + 64, c3b);
+          }
+          ++nk;
+          progress = true;
+        }
+        // V_j once K_{j+1} is out (or K is done): QK^T needs K a tile before PV needs V
+        if ((nv + 1 < nk || nk == ntiles) &&
+            (nv < NV || tc::mbar_test_wait(ve0 + 8 * (nv % NV), ((nv / NV) - 1) & 1))) {
+          const int vs = nv % NV, s0 = c0 + nv * KT;
+          const int c3a = ring[nv % CRD][0], c3b = ring[nv % CRD][1];
+          tc::mbar_arrive_expect_tx(vf0 + 8 * vs, KV_TILE);
+#pragma unroll
+          for (int r = 0; r < NR; ++r) {
+            tc::tma_load_4d(v_s(vs) + r * KV_REGION, &P.tmap_v, vf0 + 8 * vs, r * 64, g, P.paged ? 0 : s0, c3a);
+            tc::tma_load_4d(v_s(vs) + r * KV_REGION + 8192, &P.tmap_v, vf0 + 8 * vs, r * 64, g,
+                            P.paged ? 0 : s0 + 64, c3b);
+          }
+          ++nv;
+          progress = true;
+        }
+        if (progress) {
+          idle = 0;
+        } else if ((++idle & 255u) == 0) {
+          const uint64_t now = tc::global_ns();
+          if (idle == 256u) {
+            t_idle = now;
+          } else if (now - t_idle > 2000000000ull) {
+            give_up();
+            break;
           }
         }
-        const int ks = j % NK, vs = j % NV;
-        if (j >= NK && !tc::mbar_wait(ke0 + 8 * ks, ((j / NK) - 1) & 1, abort_flag)) {
-          give_up();
-          break;
-        }
-        tc::mbar_arrive_expect_tx(kf0 + 8 * ks, KV_TILE);
-#pragma unroll
-        for (int r = 0; r < NR; ++r)
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-            tc::tma_load_4d(k_s(ks) + r * KV_REGION + h * 8192, &P.tmap_k, kf0 + 8 * ks, r * 64, g, c2[h], c3[h]);
-        nk = j + 1;
-        if (j >= NV && !tc::mbar_wait(ve0 + 8 * vs, ((j / NV) - 1) & 1, abort_flag)) {
-          give_up();
-          break;
-        }
-        tc::mbar_arrive_expect_tx(vf0 + 8 * vs, KV_TILE);
-#pragma unroll
-        for (int r = 0; r < NR; ++r)
-#pragma unroll
-          for (int h = 0; h < 2; ++h)
-            tc::tma_load_4d(v_s(vs) + r * KV_REGION + h * 8192, &P.tmap_v, vf0 + 8 * vs, r * 64, g, c2[h], c3[h]);
-        nv = j + 1;
       }
       // no copy may still be landing in shared memory when the CTA ends
-      for (int j = max(0, nk - NK); j < nk; ++j) tc::mbar_wait(kf0 + 8 * (j % NK), (j / NK) & 1, &s_zero);
-      for (int j = max(0, nv - NV); j < nv; ++j) tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, &s_zero);
+      tc::mbar_wait(bq, 0, &s_zero);
+      for (int j = ::max(0, nk - NK); j < nk; ++j) tc::mbar_wait(kf0 + 8 * (j % NK), (j / NK) & 1, &s_zero);
+      for (int j = ::max(0, nv - NV); j < nv; ++j) tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, &s_zero);
     }
   } else if (warp == MMA_WARP) {
     // ---------------- MMA issuer
@@ -352,8 +468,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         tc::mma_commit(ve0 + 8 * vs);
         return true;
       };
+      bool ok = tc::mbar_wait(bq, 0, abort_flag);
+      if (!ok) give_up();
       // QK of tile j + 2 reuses the S buffer of tile j, so it follows PV_j
-      bool ok = qk(0) && (ntiles < 2 || qk(1));
+      ok = ok && qk(0) && (ntiles < 2 || qk(1));
       for (int j = 0; j < ntiles && ok; ++j) ok = pv(j) && (j + 2 >= ntiles || qk(j + 2));
       tc::mma_commit(bdrain);
       tc::mbar_wait(bdrain, 0, &s_zero);
@@ -361,9 +479,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   } else if ((warp & 3) < n_act && tree_ok) {
     // ---------------- softmax warpgroup wg: tiles wg, wg + 2, ...
     const uint32_t tl = tmem + (uint32_t(32 * (warp & 3)) << 16) + 256u * wg;
-    const unsigned long long anc = (t_row < T) ? s_anc[t_row] : 0ull;
+    const unsigned long long anc = real_row ? s_anc[t_row] : 0ull;
     const int nw = (ntiles - wg + 1) / 2;
-    float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int ii = 0; ii < nw; ++ii) {
       const int j = 2 * ii + wg;
@@ -383,13 +500,25 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const int s0 = c0 + j * KT;
       if ((s0 + KT > L) || (s0 + KT > c1)) {
         // tree columns outside the row's ancestors, and columns past this
-        // split: -inf
+        // split: -inf. The allowed columns as four 32-bit words: prefix
+        // slots (< L), the row's ancestors among the tree slots (bit a of
+        // anc is slot L + a), nothing at or past c1. Kept compact: this runs
+        // on one or two tiles of a CTA, so its code is rarely in the
+        // instruction cache.
+        uint32_t w[KT / 32];
 #pragma unroll
-        for (int c = 0; c < KT; ++c) {
-          const int col = s0 + c;
-          const bool allowed = col < c1 && (col < L || ((anc >> (col - L)) & 1ull));
-          if (!allowed) sv[c] = 0xff800000u;
+        for (int q = 0; q < KT / 32; ++q) {
+          const int cb = s0 + 32 * q;  // slot of bit 0 of this word
+          const int np = L - cb, ne = c1 - cb, sh = cb - L;
+          const uint32_t pre = np >= 32 ? 0xffffffffu : (np <= 0 ? 0u : (1u << np) - 1u);
+          const uint32_t end = ne >= 32 ? 0xffffffffu : (ne <= 0 ? 0u : (1u << ne) - 1u);
+          const uint32_t tr = (sh >= 64 || sh <= -32) ? 0u
+                              : (sh >= 0 ? uint32_t(anc >> sh) : uint32_t(anc << (-sh)));
+          w[q] = (pre | tr) & end;
         }
+#pragma unroll
+        for (int c = 0; c < KT; ++c)
+          if (!((w[c >> 5] >> (c & 31)) & 1u)) sv[c] = 0xff800000u;
       }
       // row maximum of the raw scores as a tree (scale > 0, so it commutes
       // with the scaling)
@@ -427,9 +556,15 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
       if (c1 - s0 < KT) {
         // slots past the sequence end may hold any bits (0 * NaN = NaN in the
-        // PV product): zero those V rows before the MMA reads them
-        const int first = c1 - s0, nz = (KT - first) * NR * 8;
+        // PV product): zero those V rows before the MMA reads them, once the
+        // tile's copy has landed (a later landing would undo the zeros)
         const int st = j % NV;
+        if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag))) {
+          give_up();
+          ok = false;
+          break;
+        }
+        const int first = c1 - s0, nz = (KT - first) * NR * 8;
         for (int i = 32 * (warp & 3) + lane; i < nz; i += 32 * n_act) {
           const int r = first + i / (NR * 8), rc = i % (NR * 8);
           const uint32_t dst = v_s(st) + (rc >> 3) * KV_REGION + r * 128 + ((rc & 7) << 4);
@@ -457,35 +592,34 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       give_up();
       ok = false;
     }
-    if (!ok) {
-      m_ref = -INFINITY;
-      l = 0.f;
-    }
-    s_ml[wg][row] = make_float2(m_ref, l);
+    sm_ok = ok;
   }
 
-  // ---- epilogue: the two warpgroups combine their (m, l, O); warpgroup wg
-  // writes columns [wg * D/2, (wg + 1) * D/2) of its rows
+  // ---- epilogue: the two warpgroups combine their (m, l, O) into a swizzled
+  // staging copy (row-major, 16-byte chunks XOR-ed with row & 7 so that the
+  // 32 rows of a warp hit distinct banks); then all 256 threads copy it out in
+  // row order. The rings are idle once every MMA has completed: the staging
+  // copy takes the Q region and the K ring, (m, l) the last V stage.
   if (warp < 8) {
-    if ((warp & 3) >= n_act || !tree_ok) s_ml[wg][row] = make_float2(-INFINITY, 0.f);
+    const bool act = (warp & 3) < n_act && tree_ok;
+    const bool direct = nsplit_b == 1;
+    float2 *s_ml = reinterpret_cast<float2 *>(smem + Q_BYTES + (NK + NV - 1) * KV_TILE);
+    if (act && sm_ok) s_ml[wg * ROWS + row] = make_float2(m_ref, l);
     tc::fence_before_sync();
     named_sync(1, 256);
     tc::fence_after_sync();
-    if ((warp & 3) < n_act && tree_ok && !*abort_flag) {
-      const float2 a = s_ml[0][row], c = s_ml[1][row];
+    const int64_t slot = (((int64_t(b) * p.Hkv + g) * p.nrb + rb) * p.nsplit + split) * ROWS;
+    if (act && !*abort_flag) {
+      const float2 a = s_ml[row], c = s_ml[ROWS + row];
       const float M = fmaxf(a.x, c.x);
       const float ca = (a.y > 0.f) ? tc::ex2(a.x - M) : 0.f;
       const float cb = (c.y > 0.f) ? tc::ex2(c.x - M) : 0.f;
       const float Ls = ca * a.y + cb * c.y;
-      const bool valid = grow < rows_b;
-      const int hg = grow - t_row * p.G;
-      const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + hg;
       const uint32_t lanes = tmem + (uint32_t(32 * (warp & 3)) << 16);
-      const bool direct = nsplit_b == 1;
       const float inv = direct ? 1.f / Ls : 1.f;
-      const int64_t prow =
-          (((int64_t(b) * p.Hkv + g) * p.nrb + rb) * p.nsplit + split) * ROWS + row;
-#pragma unroll
+      const uint32_t rbytes = direct ? D * 2 : D * 4;
+      const uint32_t srow = smem_base + row * rbytes;
+#pragma unroll 1
       for (int c4 = 0; c4 < D / 64; ++c4) {
         const int col = wg * (D / 2) + c4 * 32;
         uint32_t oa[32], ob[32];
@@ -500,24 +634,62 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           o[e] = (va + vb) * inv;
         }
         if (direct) {
-          if (valid) {
-            uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + col);
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              dst[e] = make_uint4(pack_bf16x2(o[8 * e + 0], o[8 * e + 1]), pack_bf16x2(o[8 * e + 2], o[8 * e + 3]),
-                                  pack_bf16x2(o[8 * e + 4], o[8 * e + 5]), pack_bf16x2(o[8 * e + 6], o[8 * e + 7]));
+          for (int e = 0; e < 4; ++e) {
+            const int ch = col / 8 + e;  // 16-byte chunk of 8 bf16
+            const uint32_t dst = srow + ((ch >> 3) << 7) + (((ch & 7) ^ (row & 7)) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst),
+                         "r"(pack_bf16x2(o[8 * e + 0], o[8 * e + 1])), "r"(pack_bf16x2(o[8 * e + 2], o[8 * e + 3])),
+                         "r"(pack_bf16x2(o[8 * e + 4], o[8 * e + 5])), "r"(pack_bf16x2(o[8 * e + 6], o[8 * e + 7]))
+                         : "memory");
           }
         } else {
-          float4 *dst = reinterpret_cast<float4 *>(p.ws_o + prow * D + col);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) dst[e] = make_float4(o[4 * e], o[4 * e + 1], o[4 * e + 2], o[4 * e + 3]);
+          for (int e = 0; e < 8; ++e) {
+            const int ch = col / 4 + e;  // 16-byte chunk of 4 floats
+            const uint32_t dst = srow + ((ch >> 3) << 7) + (((ch & 7) ^ (row & 7)) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(__float_as_uint(o[4 * e + 0])),
+                         "r"(__float_as_uint(o[4 * e + 1])), "r"(__float_as_uint(o[4 * e + 2])),
+                         "r"(__float_as_uint(o[4 * e + 3]))
+                         : "memory");
+          }
         }
       }
-      if (wg == 0) {
+      if (wg == 0 && real_row) {
         if (direct) {
-          if (valid && p.lse != nullptr) p.lse[orow] = (M + log2f(Ls)) * LN2;
+          if (p.lse != nullptr) {
+            const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + (row - (t_row - t0) * p.G);
+            p.lse[orow] = (M + log2f(Ls)) * LN2;
+          }
         } else {
-          p.ws_ml[prow] = make_float2(Ls > 0.f ? M : -INFINITY, Ls);
+          p.ws_ml[slot + row] = make_float2(Ls > 0.f ? M : -INFINITY, Ls);
+        }
+      }
+    }
+    named_sync(3, 256);
+    if (tree_ok && !*abort_flag) {
+      if (direct) {
+        constexpr int CH = D / 8;
+        for (int i = tid; i < rows_blk * CH; i += 256) {
+          const int r = i / CH, ch = i - r * CH;
+          uint4 v;
+          asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];"
+                       : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                       : "r"(smem_base + r * (D * 2) + ((ch >> 3) << 7) + (((ch & 7) ^ (r & 7)) << 4)));
+          const int tn = r / p.G;
+          const int64_t orow = (int64_t(b) * p.T_max + t0 + tn) * p.Hq + g * p.G + (r - tn * p.G);
+          *reinterpret_cast<uint4 *>(p.out + orow * D + ch * 8) = v;
+        }
+      } else {
+        constexpr int CH = D / 4;
+        float4 *dst = reinterpret_cast<float4 *>(p.ws_o + slot * D);
+        for (int i = tid; i < rows_blk * CH; i += 256) {
+          const int r = i / CH, ch = i - r * CH;
+          float4 v;
+          asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                       : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                       : "r"(smem_base + r * (D * 4) + ((ch >> 3) << 7) + (((ch & 7) ^ (r & 7)) << 4)));
+          dst[i] = v;
         }
       }
     }
@@ -536,18 +708,21 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
 
 // Log-sum-exp merge of the split partials: one warp per query row of a
 // (b, g, row block); rows of sequences that needed a single split were
-// written by the attention kernel and are skipped. Launched as a programmatic
-// dependent of the attention kernel: griddepcontrol.wait returns once that
-// grid has completed and its writes are visible.
+// written by the attention kernel and are skipped. The partial O rows of all
+// splits are loaded together with their (m, l) (a split that saw no allowed
+// key wrote zeros), so a row costs about one memory latency. Launched as a
+// programmatic dependent of the attention kernel: griddepcontrol.wait returns
+// once that grid has completed and its writes are visible.
 template <int D>
 __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  constexpr int NL = D / 4;  // lanes holding 4 columns each
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t row = int64_t(blockIdx.x) * 8 + warp;
-  const int64_t pair = row / ROWS;
-  const int r = int(row - pair * ROWS);
-  const int rb = int(pair % p.nrb);
-  const int64_t bg = pair / p.nrb;
+  const int64_t item = row / ROWS;
+  const int r = int(row - item * ROWS);
+  const int rb = int(item % p.nrb);
+  const int64_t bg = item / p.nrb;
   const int g = int(bg % p.Hkv);
   const int b = int(bg / p.Hkv);
   if (b >= p.B) return;
@@ -555,8 +730,17 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
   const int L = __ldg(p.kv_len + b);
   if (T < 1 || T > p.T_max || L < 0 || L > p.capacity - T) return;
   const int nsplit_b = (L + T + p.chunk - 1) / p.chunk;
-  const int gr = rb * ROWS + r;
-  if (nsplit_b == 1 || gr >= T * p.G) return;
+  const int t0 = rb * p.TB;
+  if (nsplit_b == 1 || t0 >= T || r >= ::min(p.TB, T - t0) * p.G) return;
+
+  const int64_t sbase = item * p.nsplit * ROWS + r;
+  float4 x[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    x[k] = (k < nsplit_b && lane < NL)
+               ? __ldcg(reinterpret_cast<const float4 *>(p.ws_o + (sbase + int64_t(k) * ROWS) * D) + lane)
+               : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float2 ml = lane < nsplit_b ? __ldcg(p.ws_ml + sbase + int64_t(lane) * ROWS) : make_float2(-INFINITY, 0.f);
   int bad = 0;  // the attention kernel skipped malformed trees; so does the merge
   for (int i = lane; i < T; i += 32) {
     const int par = __ldg(p.parent + int64_t(b) * p.T_max + i);
@@ -564,28 +748,36 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
   }
   if (__any_sync(0xffffffffu, bad)) return;
 
-  const int64_t sbase = pair * p.nsplit * ROWS;
-  float M = -INFINITY;
-  for (int s = lane; s < nsplit_b; s += 32) M = fmaxf(M, __ldcg(p.ws_ml + sbase + int64_t(s) * ROWS + r).x);
+  float M = ml.y > 0.f ? ml.x : -INFINITY;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  if (lane >= D / 4) return;
+  const float w = ml.y > 0.f ? tc::ex2(ml.x - M) : 0.f;
+  float Ls = w * ml.y;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float Ls = 0.f;
-  for (int s = 0; s < nsplit_b; ++s) {
-    const float2 ml = __ldcg(p.ws_ml + sbase + int64_t(s) * ROWS + r);
-    if (ml.y == 0.f) continue;
-    const float w = tc::ex2(ml.x - M);
-    const float4 x = __ldcg(reinterpret_cast<const float4 *>(p.ws_o + (sbase + int64_t(s) * ROWS + r) * D) + lane);
-    Ls += w * ml.y;
-    acc.x += w * x.x;
-    acc.y += w * x.y;
-    acc.z += w * x.z;
-    acc.w += w * x.w;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const float wk = __shfl_sync(0xffffffffu, w, k);
+    acc.x += wk * x[k].x;
+    acc.y += wk * x[k].y;
+    acc.z += wk * x[k].z;
+    acc.w += wk * x[k].w;
   }
+  for (int k = 8; k < nsplit_b; ++k) {
+    const float wk = __shfl_sync(0xffffffffu, w, k);
+    if (lane < NL) {
+      const float4 y = __ldcg(reinterpret_cast<const float4 *>(p.ws_o + (sbase + int64_t(k) * ROWS) * D) + lane);
+      acc.x += wk * y.x;
+      acc.y += wk * y.y;
+      acc.z += wk * y.z;
+      acc.w += wk * y.w;
+    }
+  }
+  if (lane >= NL) return;
   const float inv = 1.f / Ls;
-  const int t = gr / p.G, h = g * p.G + (gr - t * p.G);
-  const int64_t orow = (int64_t(b) * p.T_max + t) * p.Hq + h;
+  const int tn = r / p.G;
+  const int64_t orow = (int64_t(b) * p.T_max + t0 + tn) * p.Hq + g * p.G + (r - tn * p.G);
   uint2 pk;
   pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
   pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
@@ -595,10 +787,12 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
 
 // ------------------------------------------------------------------ host side
 struct AttnPlan {
+  int TB;
   int nrb;
   int nsplit;
   int chunk;
-  size_t ws_o_bytes, ws_ml_bytes;
+  bool ordered;
+  size_t ws_o_bytes, ws_ml_bytes, order_bytes;
   size_t ws_bytes;
 };
 
@@ -606,17 +800,20 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // KV splits: one CTA per SM, so pick the split count whose grid, in whole
 // waves of num_sms CTAs, gives the shortest estimated time (a wave costs its
-// chunk plus a fixed start-up of about four tiles); splits of >= 256 tokens.
+// chunk plus a fixed start-up and write-out of about four tiles: the first
+// tiles of all SMs arrive together; a merge pass about two more); splits of
+// >= 256 tokens, at most MAX_SPLITS.
 AttnPlan plan(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
   AttnPlan pl{};
   const int G = Hq / kv->Hkv;
-  pl.nrb = (tree->T_max * G + ROWS - 1) / ROWS;
+  pl.TB = std::max(1, ROWS / G);
+  pl.nrb = (tree->T_max + pl.TB - 1) / pl.TB;
   const int64_t base = int64_t(tree->B) * kv->Hkv * pl.nrb;
   const int64_t sms = num_sms();
   const int64_t max_ns = std::max<int64_t>(1, (kv->capacity + 255) / 256);
   int64_t best_ns = 1;
   double best_cost = 1e300;
-  for (int64_t ns = 1; ns <= std::min<int64_t>(max_ns, 64); ++ns) {
+  for (int64_t ns = 1; ns <= std::min<int64_t>(max_ns, MAX_SPLITS); ++ns) {
     int64_t chunk = (kv->capacity + ns - 1) / ns;
     chunk = (chunk + KT - 1) / KT * KT;
     const int64_t n = (kv->capacity + chunk - 1) / chunk;
@@ -636,14 +833,16 @@ AttnPlan plan(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
     pl.ws_o_bytes = align_up(slots * kv->D * sizeof(float), 256);
     pl.ws_ml_bytes = align_up(slots * sizeof(float2), 256);
   }
-  pl.ws_bytes = pl.ws_o_bytes + pl.ws_ml_bytes;
+  pl.ordered = tree->B > 1;
+  if (pl.ordered) pl.order_bytes = align_up(size_t(tree->B) * pl.nsplit * sizeof(int32_t), 256);
+  pl.ws_bytes = pl.ws_o_bytes + pl.ws_ml_bytes + pl.order_bytes;
   return pl;
 }
 
 bool valid_shapes(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
   return kv != nullptr && tree != nullptr && tree->B >= 1 && tree->B <= 65535 && tree->T_max >= 1 &&
          tree->T_max <= 64 && kv->Hkv >= 1 && kv->Hkv <= 65535 && Hq >= kv->Hkv && Hq % kv->Hkv == 0 &&
-         kv->capacity >= 1 && kv->n_layers >= 1;
+         Hq / kv->Hkv <= ROWS && kv->capacity >= 1 && kv->n_layers >= 1;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -688,11 +887,43 @@ bool make_kv_map(CUtensorMap *m, const void *base, const dreams_kv_cache_t *kv, 
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 5-D view of the queries, (D, G, Hkv, T_max, B), with a (64 columns, G
+// heads, 1 KV head, TB nodes, 1) box: the query rows of one row block in
+// (node, head) order, 128-byte swizzle.
+bool make_q_map(CUtensorMap *m, const void *q, int B, int T_max, int Hq, int Hkv, int D, int TB) {
+  EncodeTiledFn enc = encode_tiled();
+  if (enc == nullptr) return false;
+  const int G = Hq / Hkv;
+  const cuuint64_t dims[5] = {cuuint64_t(D), cuuint64_t(G), cuuint64_t(Hkv), cuuint64_t(T_max), cuuint64_t(B)};
+  const cuuint64_t strides[4] = {cuuint64_t(D) * 2, cuuint64_t(G) * D * 2, cuuint64_t(Hq) * D * 2,
+                                 cuuint64_t(T_max) * Hq * D * 2};
+  const cuuint32_t box[5] = {64, cuuint32_t(G), 1, cuuint32_t(TB), 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(q), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Dynamic shared memory; at least 120 KB so that one CTA runs per SM (the
 // CTA takes all 512 TMEM columns).
 template <int D>
 constexpr size_t smem_bytes() {
   return std::max<size_t>(size_t(D / 64) * ROWS * 128 + size_t(NK + NV) * (D / 64) * KT * 128 + 1024, 120 * 1024);
+}
+
+cudaError_t launch_pdl(const void *func, dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                       void **args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelExC(&cfg, func, args);
 }
 
 template <int D>
@@ -715,23 +946,29 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   memset(&P, 0, sizeof(P));
   P.a = a;
   P.paged = kv->page_table != nullptr;
-  if (!make_kv_map(&P.tmap_k, k, kv, B) || !make_kv_map(&P.tmap_v, v, kv, B)) return DREAMS_ERR_UNSUPPORTED;
-  dim3 grid(pl.nrb * pl.nsplit, a.Hkv, B);
-  tree_attn_tc_kernel<D><<<grid, THREADS, smem, stream>>>(P);
+  if (!make_kv_map(&P.tmap_k, k, kv, B) || !make_kv_map(&P.tmap_v, v, kv, B) ||
+      !make_q_map(&P.tmap_q, a.q, B, a.T_max, a.Hq, a.Hkv, D, a.TB))
+    return DREAMS_ERR_UNSUPPORTED;
+  if (pl.ordered) {
+    tree_attn_order_kernel<<<1, ORDER_THREADS, 0, stream>>>(a);
+    dreams_status_t st = check_launch();
+    if (st != DREAMS_OK) return st;
+  }
+  const int64_t ctas = int64_t(B) * pl.nsplit * a.Hkv * pl.nrb;
+  void *args_attn[] = {&P};
+  cudaError_t e = launch_pdl(reinterpret_cast<const void *>(tree_attn_tc_kernel<D>), dim3(unsigned(ctas)),
+                             dim3(THREADS), smem, stream, pl.ordered, args_attn);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
   dreams_status_t st = check_launch();
   if (st != DREAMS_OK || pl.nsplit == 1) return st;
   const int64_t rows = int64_t(B) * a.Hkv * pl.nrb * ROWS;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(unsigned((rows + 7) / 8));
-  cfg.blockDim = dim3(256);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, tree_attn_merge_kernel<D>, a);
+  AttnParams am = a;
+  void *args_merge[] = {&am};
+  e = launch_pdl(reinterpret_cast<const void *>(tree_attn_merge_kernel<D>), dim3(unsigned((rows + 7) / 8)),
+                 dim3(256), 0, stream, true, args_merge);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return DREAMS_ERR_CUDA;
@@ -774,7 +1011,7 @@ extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_k
   const AttnPlan pl = plan(kv, tree, Hq);
   if (pl.ws_bytes > 0 && (workspace == nullptr || workspace_bytes < pl.ws_bytes || !aligned16(workspace)))
     return DREAMS_ERR_WORKSPACE;
-  if (int64_t(pl.nrb) * pl.nsplit > 0x7fffffff) return DREAMS_ERR_UNSUPPORTED;
+  if (int64_t(tree->B) * pl.nsplit * kv->Hkv * pl.nrb > 0x7fffffff) return DREAMS_ERR_UNSUPPORTED;
 
   AttnParams p{};
   p.q = static_cast<const __nv_bfloat16 *>(q);
@@ -792,15 +1029,17 @@ extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_k
   p.Hq = Hq;
   p.Hkv = kv->Hkv;
   p.G = Hq / kv->Hkv;
+  p.TB = pl.TB;
   p.nrb = pl.nrb;
   p.nsplit = pl.nsplit;
   p.chunk = pl.chunk;
   p.scale_log2 = scale * LOG2E;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
-  if (pl.ws_bytes > 0) {
+  if (pl.nsplit > 1) {
     p.ws_o = reinterpret_cast<float *>(ws);
     p.ws_ml = reinterpret_cast<float2 *>(ws + pl.ws_o_bytes);
   }
+  if (pl.ordered) p.order = reinterpret_cast<int32_t *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes);
   p.status = status_word;
   const void *k = static_cast<const __nv_bfloat16 *>(kv->k) + int64_t(layer) * kv->layer_stride;
   const void *v = static_cast<const __nv_bfloat16 *>(kv->v) + int64_t(layer) * kv->layer_stride;

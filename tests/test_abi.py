@@ -52,6 +52,8 @@ def test_workspace_sizes(lib):
     n = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 32)
     assert n > 0 and n % 256 == 0
     tr = dreams._Tree(16, 16, 16, 16, 16, 64)
+    # several sequences: the longest-first order of the work items needs room too
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32) >= 16 * 4
     bad = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
     assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(bad), ctypes.byref(tr), 30) == 0
     assert lib.dreams_vocab_argmax_workspace_size(768, 128256) >= 0
@@ -76,6 +78,7 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert attn(out=null) == dreams.ERR_INVALID_ARG
     assert attn(q=P + 2) == dreams.ERR_INVALID_ARG           # misaligned
     assert attn(Hq=3) == dreams.ERR_INVALID_ARG              # Hq % Hkv
+    assert attn(Hq=258) == dreams.ERR_INVALID_ARG            # more than 128 query heads per KV head
     assert attn(layer=1) == dreams.ERR_INVALID_ARG
     assert attn(scale=float("inf")) == dreams.ERR_INVALID_ARG
     assert attn(tree=dreams._Tree(P, P, P, P, 2, 65)) == dreams.ERR_INVALID_ARG   # T_max > 64

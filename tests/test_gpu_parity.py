@@ -73,6 +73,9 @@ def test_attention_mask_sensitive(dreams, name, L, key_scale):
     (2, 8, 2, 128, 17, 63, 200),   # ragged tile boundary
     (3, 4, 4, 64, 64, 129, 400),   # maximum tree
     (2, 16, 2, 128, 64, 1000, 1100),  # 512 query rows per KV head: several row blocks
+    (2, 14, 2, 128, 40, 300, 400),    # group of 7 heads: 18 nodes (126 rows) per row block
+    (1, 100, 1, 64, 5, 100, 200),     # group of 100 heads: one node per row block
+    (2, 128, 1, 64, 3, 50, 100),      # the largest group (128 heads)
 ])
 def test_attention_edge_shapes(dreams, B, Hq, Hkv, D, T, L, cap):
     rng = np.random.default_rng(B * 1000 + T)
@@ -101,6 +104,33 @@ def test_attention_edge_shapes(dreams, B, Hq, Hkv, D, T, L, cap):
     assert (out[-1, tl[-1]:].float() == 7.0).all()
 
 
+def test_attention_uneven_lengths(dreams):
+    """Sequences of very different lengths in one call: the long ones are
+    split over several CTAs and merged, the short ones are not, and the
+    items run longest first."""
+    rng = np.random.default_rng(77)
+    B, Hq, Hkv, D, T, cap = 5, 8, 2, 128, 24, 4096
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    tl = np.array([24, 1, 17, 24, 9], np.int32)
+    for b in range(B):
+        par[b, tl[b]:] = -1
+    kl = np.array([4000, 0, 1500, 63, 3333], np.int32)
+    kl = np.minimum(kl, cap - tl)
+    q = W.bf16(rng.standard_normal((B, T, Hq, D), dtype=np.float32))
+    k = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    v = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    scale = 1.0 / np.sqrt(D)
+    kv = dreams.KVCache(k.cuda(), v.cuda())
+    tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
+                       torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    st = _status()
+    out, lse = dreams.tree_verify_attn(q.cuda(), kv, tree, scale, want_lse=True, status=st)
+    ref, ref_lse, sel, ost = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v), oracle.KVLayout(cap, Hkv, D),
+                                                   par, tl, kl, Hq, scale)
+    assert ost == 0 and int(st.item()) == 0
+    compare_attention(out, lse, ref, ref_lse, sel)
+
+
 def test_attention_paged_equals_contiguous(dreams):
     """The batched workload copied into a contiguous cache gives bit-identical
     results to its paged form."""
@@ -126,7 +156,7 @@ def test_attention_paged_equals_contiguous(dreams):
 
 def test_attention_repeatable(dreams):
     """Two calls on the same inputs give identical bits (the split merge has a
-    fixed order and the workspace counters reset themselves)."""
+    fixed order, whichever SM computed each split)."""
     w = W.make("long13b", with_logits=False)
     g = to_gpu(w)
     a, la = dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, want_lse=True)
