@@ -182,6 +182,8 @@ def run_dreams(args, rank, world, local):
                           dtype=torch.uint8, device=dev)
     ws_step = torch.zeros(dreams.verify_step_workspace_size(copies[0]["tree"], w.V), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
+    launches_per_step = (dreams.tree_verify_attn_launches(copies[0]["kv"], copies[0]["tree"], w.Hq)
+                         + dreams.VERIFY_STEP_LAUNCHES)
 
     def step(c, ev=None):
         if ev is not None:
@@ -305,7 +307,7 @@ def run_dreams(args, rank, world, local):
                        "kv_tokens": int((w.kv_len + w.tree_len).sum()), "tree_nodes": int(w.tree_len.sum()),
                        "l2": f"inputs larger than L2: 2 rotating copies of {copy_bytes / 2**20:.0f} MiB each",
                        "parallelism": f"replicas x{world}"},
-            "e2e": e2e, "gpu_launches": 2 * K, "roofline": roofline, "kernels": kernels,
+            "e2e": e2e, "gpu_launches": launches_per_step * K, "roofline": roofline, "kernels": kernels,
             "tau_mean_accept_len": None, "clocks": clk, "cpu_baseline": cpu, "wall_s": round(wall, 3),
         }
         acc = copies[0]["outs"][0].float().mean().item()

@@ -19,7 +19,7 @@
  *                               the target's bonus token;
  *   4. dreams_kv_compact        the accepted nodes' K/V moved into contiguous
  *                               cache slots for the next step;
- *   5. dreams_verify_step       2 + 3 + 4 in one launch.
+ *   5. dreams_verify_step       2 + 3 + 4 in one call (two launches).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -136,6 +136,10 @@ typedef struct dreams_tree {
  */
 size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
                                               int32_t Hq);
+/* Kernel launches one dreams_tree_verify_attn call with these shapes makes
+ * (1 to 3: an ordering pass for B > 1, the attention, a merge of the KV
+ * splits when the cache is split); 0 for shapes the call rejects. */
+int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int32_t Hq);
 dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
                                         const dreams_tree_t *tree, int32_t Hq, float scale, void *out,
                                         float *lse, void *workspace, size_t workspace_bytes,
@@ -189,12 +193,14 @@ dreams_status_t dreams_kv_compact(const dreams_kv_cache_t *kv, int32_t B, const 
                                   int32_t *status_word, dreams_stream_t stream);
 
 /*
- * The verification tail in one launch: dreams_vocab_argmax over the rows of
+ * The verification tail in one call: dreams_vocab_argmax over the rows of
  * tree nodes (row b * T_max + i for i < tree_len[b]; logits [B, T_max, V]
  * with row_stride), then dreams_accept_path, then dreams_kv_compact on all
  * kv->n_layers layers, with the semantics documented above. argmax_out
  * ([B, T_max], may be NULL) receives the predictions of the rows computed;
- * other rows are untouched.
+ * other rows are untouched. The call makes two kernel launches on the
+ * stream: the argmax, then the walk and compaction (one CTA per sequence),
+ * chained by programmatic dependent launch.
  */
 size_t dreams_verify_step_workspace_size(const dreams_tree_t *tree, int64_t V);
 dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int64_t V,

@@ -76,6 +76,7 @@ def _lib() -> ctypes.CDLL:
                 pkv, ptr = ctypes.POINTER(_KVCache), ctypes.POINTER(_Tree)
                 sig = {
                     "dreams_tree_verify_attn_workspace_size": (sz, [pkv, ptr, i32]),
+                    "dreams_tree_verify_attn_launches": (i32, [pkv, ptr, i32]),
                     "dreams_tree_verify_attn": (ctypes.c_int, [p, pkv, i32, ptr, i32, f32, p, p, p, sz, p, p]),
                     "dreams_vocab_argmax_workspace_size": (sz, [i64, i64]),
                     "dreams_vocab_argmax": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p, sz, p]),
@@ -217,6 +218,14 @@ def tree_verify_attn_workspace_size(kv: KVCache, tree: Tree, Hq: int) -> int:
     return int(_lib().dreams_tree_verify_attn_workspace_size(ctypes.byref(kv._c), ctypes.byref(tree._c), Hq))
 
 
+def tree_verify_attn_launches(kv: KVCache, tree: Tree, Hq: int) -> int:
+    """Kernel launches one tree_verify_attn call with these shapes makes."""
+    return int(_lib().dreams_tree_verify_attn_launches(ctypes.byref(kv._c), ctypes.byref(tree._c), Hq))
+
+
+VERIFY_STEP_LAUNCHES = 2  # dreams_verify_step: the argmax, then the walk and compaction
+
+
 def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, layer: int = 0,
                      out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
                      want_lse: bool = False, workspace: Optional[torch.Tensor] = None,
@@ -326,7 +335,7 @@ def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
                 workspace: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
                 stream=None) -> dict:
     """Argmax of the tree rows of ``logits`` ([B, T_max, V] f32/bf16), greedy
-    acceptance and KV compaction, in one launch."""
+    acceptance and KV compaction, in one call (two kernel launches)."""
     dev = tree.parent.device
     if logits.dtype not in (torch.float32, torch.bfloat16) or logits.device != dev:
         raise TypeError("logits must be float32/bfloat16 on the tree's device")

@@ -987,6 +987,13 @@ extern "C" size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t
   return plan(kv, tree, Hq).ws_bytes;
 }
 
+extern "C" int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
+                                                    int32_t Hq) {
+  if (!valid_shapes(kv, tree, Hq) || (kv->D != 64 && kv->D != 128)) return 0;
+  const AttnPlan pl = plan(kv, tree, Hq);
+  return 1 + (pl.ordered ? 1 : 0) + (pl.nsplit > 1 ? 1 : 0);
+}
+
 extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
                                                    const dreams_tree_t *tree, int32_t Hq, float scale,
                                                    void *out, float *lse, void *workspace,

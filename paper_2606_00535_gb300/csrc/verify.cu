@@ -23,6 +23,11 @@
 // from the walk starts at 0 and increases, so source slot path[x] >= x and a
 // thread that reads its sources before writing them (batches of 8, batch by
 // batch in increasing x) never overwrites a slot it still has to read.
+//
+// The fused step is two launches: the argmax over the rows of real tree nodes,
+// then, one CTA per sequence and chained by programmatic dependent launch, the
+// walk and the compaction. Kept apart, the argmax kernel needs few registers,
+// so every CTA of a large batch is resident at once.
 #include <limits.h>
 
 #include <algorithm>
@@ -489,75 +494,65 @@ struct StepParams {
   int32_t max_path;
   int32_t *pred;  // [B, T_max] predictions (caller's argmax_out or workspace)
   bool pred_in_ws;
-  int32_t *seq_cnt;
   int32_t *accept_len, *path, *out_tokens, *new_kv_len;
   int32_t *status;
 };
 
-// grid.x = B * T_max * nchunk: (sequence, tree node, vocabulary chunk).
+// Launch 1 of the verification tail. grid.x = B * T_max * nchunk: (sequence,
+// tree node, vocabulary chunk); CTAs of padding nodes return at once. The CTA
+// that completes a node's row writes the node's prediction.
 template <typename T>
-__global__ void __launch_bounds__(TAIL_THREADS) verify_step_kernel(const StepParams p) {
-  __shared__ int32_t s_path[65];
-  __shared__ int64_t s_src[65], s_dst[65];
-  __shared__ int s_go;
+__global__ void __launch_bounds__(ARGMAX_THREADS) verify_rows_kernel(const StepParams p) {
+  // the walk kernel may start now: it waits for this grid to complete
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int nchunk = p.am.nchunk;
   const int c = blockIdx.x % nchunk;
   const int rowg = blockIdx.x / nchunk;
   const int b = rowg / p.tr.T_max, i = rowg % p.tr.T_max;
   const int tl = __ldg(p.tr.tree_len + b);
-  const int L = __ldg(p.tr.kv_len + b);
+  if (tl < 1 || tl > p.tr.T_max || i >= tl) return;
   const int64_t rb = int64_t(b) * p.tr.T_max;
-  if (tl < 1 || tl > p.tr.T_max) {
-    if (i == 0 && c == 0 && threadIdx.x < 32) {
-      if (threadIdx.x == 0) flag(p.status, DREAMS_DATA_BAD_TREE_LEN);
-      write_walk(b, -1, L, p.tr.tokens + rb, p.pred + rb, s_path, p.max_path, p.accept_len, p.path, p.out_tokens,
-                 p.new_kv_len);
-    }
-    return;
-  }
-  if (i >= tl) return;
-
-  // -- argmax of row (b, i), chunk c
   const T *row = static_cast<const T *>(p.am.logits) + (rb + i) * p.am.row_stride;
   const int64_t begin = c * p.am.chunk, end = std::min<int64_t>(p.am.V, begin + p.am.chunk);
   int key, idx, row_idx;
   block_argmax<T>(row, begin, end, p.am.vec_ok, key, idx);
-  if (!row_combine(nchunk, p.am.slot + rb + i, p.am.cnt + rb + i, key, idx, row_idx)) return;
-
-  // -- this CTA finished row (b, i); the last row of sequence b runs the tail
-  if (threadIdx.x == 0) {
+  if (row_combine(nchunk, p.am.slot + rb + i, p.am.cnt + rb + i, key, idx, row_idx) && threadIdx.x == 0)
     p.pred[rb + i] = row_idx;
-    __threadfence();
-    const int last = atomicAdd(p.seq_cnt + b, 1) == tl - 1;
-    if (last) {
-      p.seq_cnt[b] = 0;
-      __threadfence();
-    }
-    s_go = last;
-  }
-  __syncthreads();
-  if (!s_go) return;
+}
 
+// Launch 2 of the verification tail, one CTA per sequence, chained to launch 1
+// by programmatic dependent launch (it may start early and waits until launch
+// 1 has completed): the acceptance walk, its outputs, and the KV compaction.
+__global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepParams p) {
+  __shared__ int32_t s_path[65];
+  __shared__ int64_t s_src[65], s_dst[65];
+  __shared__ int s_n;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int b = blockIdx.x, Tm = p.tr.T_max;
+  const int64_t rb = int64_t(b) * Tm;
+  const int T = __ldg(p.tr.tree_len + b);
+  const int L = __ldg(p.tr.kv_len + b);
   if (threadIdx.x < 32) {
     WalkOut w{-1, 0};
-    if (L < 0 || L > p.kv.capacity - tl) w.bad = DREAMS_DATA_BAD_KV_LEN;
-    else w = tree_walk_warp(p.tr.parent + rb, p.tr.tokens + rb, p.pred + rb, tl, p.max_path, s_path);
+    if (T < 1 || T > Tm) w.bad = DREAMS_DATA_BAD_TREE_LEN;
+    else if (L < 0 || L > p.kv.capacity - T) w.bad = DREAMS_DATA_BAD_KV_LEN;
+    else w = tree_walk_warp(p.tr.parent + rb, p.tr.tokens + rb, p.pred + rb, T, p.max_path, s_path);
     if (w.bad) {
       w.n = -1;
       if (threadIdx.x == 0) flag(p.status, w.bad);
     }
     write_walk(b, w.n, L, p.tr.tokens + rb, p.pred + rb, s_path, p.max_path, p.accept_len, p.path, p.out_tokens,
                p.new_kv_len);
-    if (p.pred_in_ws) {  // leave the workspace zero-filled
+    if (p.pred_in_ws && T >= 1 && T <= Tm) {  // leave the workspace zero-filled
       __syncwarp();
-      for (int x = threadIdx.x; x < tl; x += 32) p.pred[rb + x] = 0;
+      for (int x = threadIdx.x; x < T; x += 32) p.pred[rb + x] = 0;
     }
     bool ok = w.n > 0;
     if (ok) ok = move_offsets(p.kv, b, L, w.n, s_path, s_src, s_dst, p.status);
-    if (threadIdx.x == 0) s_go = ok ? w.n : 0;
+    if (threadIdx.x == 0) s_n = ok ? w.n : 0;
   }
   __syncthreads();
-  const int n = s_go;
+  const int n = s_n;
   if (n > 0) compact_units(p.kv, n, s_src, s_dst, threadIdx.x, blockDim.x);
 }
 
@@ -683,7 +678,7 @@ extern "C" dreams_status_t dreams_kv_compact(const dreams_kv_cache_t *kv, int32_
 extern "C" size_t dreams_verify_step_workspace_size(const dreams_tree_t *tree, int64_t V) {
   if (tree == nullptr || tree->B < 1 || tree->T_max < 1 || V < 1) return 0;
   const int64_t rows = int64_t(tree->B) * tree->T_max;
-  return argmax_ws(rows) + align_up(size_t(rows) * 4, 256) + align_up(size_t(tree->B) * 4, 256);
+  return argmax_ws(rows) + align_up(size_t(rows) * 4, 256);
 }
 
 extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int64_t V,
@@ -715,7 +710,6 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   p.am.slot = reinterpret_cast<unsigned long long *>(ws);
   p.am.cnt = reinterpret_cast<int32_t *>(ws + align_up(size_t(rows) * 8, 256));
   int32_t *ws_pred = reinterpret_cast<int32_t *>(ws + argmax_ws(rows));
-  p.seq_cnt = reinterpret_cast<int32_t *>(ws + argmax_ws(rows) + align_up(size_t(rows) * 4, 256));
   p.pred = argmax_out != nullptr ? argmax_out : ws_pred;
   p.pred_in_ws = argmax_out == nullptr;
   p.max_path = max_path;
@@ -726,8 +720,24 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   p.status = status_word;
   const dim3 grid(unsigned(rows * pl.nchunk));
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (dtype == DREAMS_F32) verify_step_kernel<float><<<grid, TAIL_THREADS, 0, s>>>(p);
-  else verify_step_kernel<__nv_bfloat16><<<grid, TAIL_THREADS, 0, s>>>(p);
+  if (dtype == DREAMS_F32) verify_rows_kernel<float><<<grid, ARGMAX_THREADS, 0, s>>>(p);
+  else verify_rows_kernel<__nv_bfloat16><<<grid, ARGMAX_THREADS, 0, s>>>(p);
+  dreams_status_t st = check_launch();
+  if (st != DREAMS_OK) return st;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(tree->B));
+  cfg.blockDim = dim3(TAIL_THREADS);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_tail_kernel, p);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
   return check_launch();
 }
 

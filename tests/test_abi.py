@@ -60,6 +60,21 @@ def test_workspace_sizes(lib):
     assert lib.dreams_verify_step_workspace_size(ctypes.byref(tr), 128256) >= 16 * 64 * 16
 
 
+def test_attention_launch_count(lib):
+    """One sequence: the attention, plus a merge when the KV range is split
+    (the workspace then holds the partials); several sequences add the
+    longest-first ordering pass; rejected shapes make no launch."""
+    kvc = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
+    one = dreams._Tree(16, 16, 16, 16, 1, 64)
+    split = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 32) > 0
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(one), 32) == 1 + int(split)
+    many = dreams._Tree(16, 16, 16, 16, 16, 64)
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(many), 32) >= 2
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(many), 30) == 0
+    d96 = dreams._KVCache(16, 16, 1, 0, 8, 96, 6080, None, 0, 0, 0)
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(d96), ctypes.byref(many), 32) == 0
+
+
 @pytest.mark.skipif(torch.cuda.is_available(), reason="host-validation cases use placeholder pointers")
 def test_invalid_arguments_rejected_before_launch(lib):
     """Each case breaks exactly one rule and must be refused on the host."""

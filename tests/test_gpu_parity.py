@@ -383,3 +383,93 @@ def test_status_word_clean_on_valid_input(dreams):
     dreams.tree_verify_attn(g["q"], g["kv"], g["tree"], w.scale, status=st)
     dreams.verify_step(g["logits"], g["tree"], g["kv"], w.max_path, status=st)
     assert int(st.item()) == 0
+
+
+# ------------------------------------------------------------------ scan partition
+def test_argmax_many_short_rows(dreams):
+    """More rows than eight per CTA: every CTA takes whole rows (no workspace)."""
+    rows, V = 5003, 37
+    rng = np.random.default_rng(11)
+    x = (rng.standard_normal((rows, V)) * 2).astype(np.float32)
+    x[::7, 5] = x[::7, 30] = 99.0  # ties inside a row
+    assert dreams._lib().dreams_vocab_argmax_workspace_size(rows, V) == 0
+    for t in (torch.from_numpy(x), torch.from_numpy(x).to(torch.bfloat16)):
+        ref = (oracle.argmax(W.bits(t), bf16_bits=True) if t.dtype == torch.bfloat16 else oracle.argmax(x))
+        np.testing.assert_array_equal(dreams.vocab_argmax(t.cuda()).cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_argmax_split_rows_repeat(dreams, dtype):
+    """Rows split between many CTAs, aligned and unaligned bases, two calls on
+    one explicit workspace: same answers, workspace zero-filled afterwards."""
+    rows, V = 5, 300_001
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((rows, V)).astype(np.float32)
+    x[0, [17, 250_000]] = 40.0   # equal maxima far apart: lowest index wins
+    x[1, V - 1] = 40.0           # the maximum in the partial last vector
+    x[2, 123_457] = float("nan")
+    t = torch.from_numpy(x).to(dtype)
+    ref = (oracle.argmax(W.bits(t), bf16_bits=True) if dtype == torch.bfloat16 else oracle.argmax(x))
+    need = dreams._lib().dreams_vocab_argmax_workspace_size(rows, V)
+    assert need > 0
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    pad = torch.zeros((rows, V + 3), dtype=dtype)
+    pad[:, 1:V + 1] = t
+    for src in (t.cuda(), pad.cuda()[:, 1:V + 1]):
+        for _ in range(2):
+            got = dreams.vocab_argmax(src, workspace=ws)
+            np.testing.assert_array_equal(got.cpu().numpy(), ref)
+            assert int(ws.count_nonzero().item()) == 0
+
+
+@pytest.mark.parametrize("dtype,aligned", [(torch.bfloat16, True), (torch.float32, False)])
+def test_verify_step_ragged_repeat(dreams, dtype, aligned):
+    """Ragged and invalid trees, a vocabulary that is not a multiple of the
+    vector width, rows split between CTAs; two calls on one workspace."""
+    rng = np.random.default_rng(13)
+    B, T_max, V, Hkv, D, cap = 7, 9, 100_003, 2, 16, 64
+    tl = np.array([1, 9, 0, 5, 9, 2, 3], np.int32)  # sequence 2 is invalid
+    par = np.full((B, T_max), -1, np.int32)
+    for b in range(B):
+        if tl[b] > 0:
+            par[b, :tl[b]] = W.random_tree(rng, int(tl[b]))
+    tok = rng.integers(0, V, (B, T_max)).astype(np.int32)
+    x = rng.standard_normal((B, T_max, V)).astype(np.float32)
+    for b in range(B):  # plant matches along the first child of each node
+        for i in range(1, int(tl[b])):
+            x[b, par[b, i], tok[b, i]] = 50.0 + i
+    kl = np.array([0, 10, 5, 40, 55, 3, 20], np.int32)
+    k = torch.from_numpy(rng.standard_normal((B, cap, Hkv, D)).astype(np.float32)).to(torch.bfloat16)
+    v = torch.from_numpy(rng.standard_normal((B, cap, Hkv, D)).astype(np.float32)).to(torch.bfloat16)
+    t = torch.from_numpy(x).to(dtype)
+    rows_ref = (oracle.argmax(W.bits(t.reshape(-1, V)), bf16_bits=True) if dtype == torch.bfloat16
+                else oracle.argmax(x.reshape(-1, V))).reshape(B, T_max)
+    ref = oracle.accept_path(rows_ref, par, tok, tl, kl, T_max + 1)
+    if aligned:
+        lg = t.cuda()
+    else:
+        pad = torch.zeros((B, T_max, V + 1), dtype=dtype)
+        pad[:, :, 1:] = t
+        lg = pad.cuda()[:, :, 1:]
+    f = lambda a: torch.as_tensor(a).cuda()
+    tree = dreams.Tree(f(par), f(tok), f(tl), f(kl))
+    kv = dreams.KVCache(k.cuda(), v.cuda())
+    ws = torch.zeros(dreams.verify_step_workspace_size(tree, V), dtype=torch.uint8, device="cuda")
+    lay = oracle.KVLayout(cap, Hkv, D)
+    ko, vo = W.bits(k), W.bits(v)
+    for call in range(2):
+        st = _status()
+        am = torch.full((B, T_max), -7, dtype=torch.int32, device="cuda")
+        r = dreams.verify_step(lg, tree, kv, T_max + 1, argmax_out=am, workspace=ws, status=st)
+        torch.cuda.synchronize()
+        assert int(st.item()) == dreams.DATA_BAD_TREE_LEN
+        assert int(ws.count_nonzero().item()) == 0
+        amc = am.cpu().numpy()
+        for b in range(B):
+            np.testing.assert_array_equal(amc[b, :tl[b]], rows_ref[b, :tl[b]])
+            assert (amc[b, tl[b]:] == -7).all()
+        for key in ("accept_len", "path", "out_tokens", "new_kv_len"):
+            np.testing.assert_array_equal(r[key].cpu().numpy(), ref[key], err_msg=key)
+        ko, vo, ost = oracle.kv_compact(ko, vo, lay, kl, ref["accept_len"], ref["path"])
+        assert ost == 0
+        assert np.array_equal(W.bits(kv.k.cpu()), ko) and np.array_equal(W.bits(kv.v.cpu()), vo)
