@@ -115,6 +115,31 @@ __device__ __forceinline__ void named_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// Three-input maximum, and f32 pairs for the packed (f32x2) FMA and add.
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f32x2_split(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // KV tiles of split s of sequence b (0 for an empty split or bad lengths).
 __device__ __forceinline__ int split_tiles(const AttnParams &p, int b, int s) {
   const int T = __ldg(p.tree_len + b);
@@ -431,6 +456,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   } else if (warp == MMA_WARP) {
     // ---------------- MMA issuer
     if (lane == 0 && tree_ok) {
+      // Base descriptors: an operand's descriptor is its base plus its byte
+      // offset / 16 (the address field holds bits 4-17 of a shared-memory
+      // address below 256 KB, so the addition never carries out of it); each
+      // MMA then costs one add.
+      const uint64_t qd0 = tc::smem_desc_sw128(q_s, 16, 1024);
+      const uint64_t kd0 = tc::smem_desc_sw128(k_s(0), 16, 1024);
+      const uint64_t vd0 = tc::smem_desc_sw128(v_s(0), KV_REGION, 1024);
       // S_j = Q K_j^T into warpgroup (j % 2)'s S buffer
       auto qk = [&](int j) {
         const int ks = j % NK;
@@ -443,8 +475,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
 #pragma unroll
         for (int k = 0; k < D / 16; ++k) {
           const uint32_t off = (k & 3) << 5;  // 32 bytes per 16-element K step
-          const uint64_t ad = tc::smem_desc_sw128(q_s + (k >> 2) * Q_REGION + off, 16, 1024);
-          const uint64_t bd = tc::smem_desc_sw128(k_s(ks) + (k >> 2) * KV_REGION + off, 16, 1024);
+          const uint64_t ad = qd0 + (((k >> 2) * Q_REGION + off) >> 4);
+          const uint64_t bd = kd0 + ((uint32_t(ks) * KV_TILE + (k >> 2) * KV_REGION + off) >> 4);
           tc::mma_ss(tmem + scol, ad, bd, IDESC_QK, k > 0 ? 1u : 0u);
         }
         tc::mma_commit(bs0 + 8 * (j & 1));
@@ -462,7 +494,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         const uint32_t scol = 256u * w, ocol = 256u * w + 128u;
 #pragma unroll
         for (int ks = 0; ks < KT / 16; ++ks) {
-          const uint64_t bd = tc::smem_desc_sw128(v_s(vs) + ks * 2048, KV_REGION, 1024);
+          const uint64_t bd = vd0 + ((uint32_t(vs) * KV_TILE + ks * 2048) >> 4);
           tc::mma_ts(tmem + ocol, tmem + scol + ks * 8, bd, IDESC_PV, (ii > 0 || ks > 0) ? 1u : 0u);
         }
         tc::mma_commit(ve0 + 8 * vs);
@@ -520,18 +552,19 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         for (int c = 0; c < KT; ++c)
           if (!((w[c >> 5] >> (c & 31)) & 1u)) sv[c] = 0xff800000u;
       }
-      // row maximum of the raw scores as a tree (scale > 0, so it commutes
-      // with the scaling)
-      float mt[32];
+      // row maximum of the raw scores as a tree of three-input maxima (scale
+      // > 0, so it commutes with the scaling)
+      float mt[43];
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        mt[i] = fmaxf(fmaxf(__uint_as_float(sv[4 * i]), __uint_as_float(sv[4 * i + 1])),
-                      fmaxf(__uint_as_float(sv[4 * i + 2]), __uint_as_float(sv[4 * i + 3])));
+      for (int i = 0; i < 42; ++i)
+        mt[i] = max3f(__uint_as_float(sv[3 * i]), __uint_as_float(sv[3 * i + 1]), __uint_as_float(sv[3 * i + 2]));
+      mt[42] = fmaxf(__uint_as_float(sv[126]), __uint_as_float(sv[127]));
 #pragma unroll
-      for (int w2 = 16; w2 > 0; w2 >>= 1)
+      for (int i = 0; i < 14; ++i) mt[i] = max3f(mt[3 * i], mt[3 * i + 1], mt[3 * i + 2]);
+      mt[14] = mt[42];  // 15 left
 #pragma unroll
-        for (int i = 0; i < w2; ++i) mt[i] = fmaxf(mt[i], mt[i + w2]);
-      const float mx = mt[0] * p.scale_log2;
+      for (int i = 0; i < 5; ++i) mt[i] = max3f(mt[3 * i], mt[3 * i + 1], mt[3 * i + 2]);
+      const float mx = max3f(max3f(mt[0], mt[1], mt[2]), mt[3], mt[4]) * p.scale_log2;
       const bool resc = mx > m_ref + RESCALE;
       float corr = 1.f;
       if (resc) {
@@ -540,20 +573,31 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         l *= corr;
       }
       const float nmu = (m_ref == -INFINITY) ? 0.f : -m_ref;
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      // exponents scale * s - m two at a time (f32x2 FMA), their sum two at a
+      // time (f32x2 add), P as bf16 pairs
+      const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2), nmu2 = f32x2(nmu, nmu);
+      uint64_t acc2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
 #pragma unroll
       for (int q4 = 0; q4 < KT / 32; ++q4) {
         uint32_t pk[16];
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
-          const float p0 = tc::ex2(fmaf(__uint_as_float(sv[32 * q4 + 2 * c]), p.scale_log2, nmu));
-          const float p1 = tc::ex2(fmaf(__uint_as_float(sv[32 * q4 + 2 * c + 1]), p.scale_log2, nmu));
-          acc[c & 3] += p0 + p1;
+          float e0, e1;
+          f32x2_split(ffma2(f32x2(__uint_as_float(sv[32 * q4 + 2 * c]), __uint_as_float(sv[32 * q4 + 2 * c + 1])),
+                            scale2, nmu2),
+                      e0, e1);
+          const float p0 = tc::ex2(e0), p1 = tc::ex2(e1);
+          acc2[c & 1] = fadd2(acc2[c & 1], f32x2(p0, p1));
           pk[c] = pack_bf16x2(p0, p1);
         }
         tc::tmem_st16(tl + 16 * q4, pk);  // P (bf16 pairs) over the first 64 columns of S
       }
-      l += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      {
+        float a0, a1, b0, b1;
+        f32x2_split(acc2[0], a0, a1);
+        f32x2_split(acc2[1], b0, b1);
+        l += (a0 + a1) + (b0 + b1);
+      }
       if (c1 - s0 < KT) {
         // slots past the sequence end may hold any bits (0 * NaN = NaN in the
         // PV product): zero those V rows before the MMA reads them, once the

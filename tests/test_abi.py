@@ -60,6 +60,17 @@ def test_workspace_sizes(lib):
     assert lib.dreams_verify_step_workspace_size(ctypes.byref(tr), 128256) >= 16 * 64 * 16
 
 
+def test_attention_workspace_covers_every_row_block(lib):
+    """A CTA takes a pair of row blocks, but the split partials are kept per
+    row block: with 5 query heads per KV head and 64 nodes there are 3 row
+    blocks (25 nodes each), so one split needs 3 x 128 rows of (O, m, l)."""
+    kvc = dreams._KVCache(16, 16, 1, 0, 1, 128, 2304, None, 0, 0, 0)
+    one = dreams._Tree(16, 16, 16, 16, 1, 64)
+    ws = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 5)
+    per_split = 3 * 128 * (128 * 4 + 8)
+    assert ws > 0 and ws % per_split == 0, ws
+
+
 def test_attention_launch_count(lib):
     """One sequence: the attention, plus a merge when the KV range is split
     (the workspace then holds the partials); several sequences add the

@@ -76,6 +76,10 @@ def test_attention_mask_sensitive(dreams, name, L, key_scale):
     (2, 14, 2, 128, 40, 300, 400),    # group of 7 heads: 18 nodes (126 rows) per row block
     (1, 100, 1, 64, 5, 100, 200),     # group of 100 heads: one node per row block
     (2, 128, 1, 64, 3, 50, 100),      # the largest group (128 heads)
+    (1, 3, 1, 128, 64, 2000, 2304),   # 2 row blocks in one CTA, KV range split
+    (1, 5, 1, 128, 64, 2000, 2304),   # 3 row blocks: a pair and a lone block, KV range split
+    (1, 6, 1, 128, 64, 2000, 2304),   # 4 row blocks: two pairs, KV range split
+    (2, 10, 2, 64, 61, 1500, 1600),   # head dim 64, pairs, ragged split tail
 ])
 def test_attention_edge_shapes(dreams, B, Hq, Hkv, D, T, L, cap):
     rng = np.random.default_rng(B * 1000 + T)
