@@ -16,6 +16,10 @@ paper passage its C routine follows:
   Sec. 3.2: attention = softmax(Q K^T / sqrt(z))).
 * :func:`argmax` -- the target's greedy (temperature 0) prediction per node
   (Sec. 2 "Speculative decoding"; Table 2, Temperature = 0).
+* :func:`sample` -- the target's own sample per node at temperature tau > 0,
+  by inverse transform of softmax(x / tau) with a caller-supplied uniform
+  (Sec. 2 "Speculative decoding": drafts are checked against the target's own
+  sampling; Table 2, Temperature = 1).
 * :func:`accept_path` -- sequential acceptance with the target's token
   replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
 * :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
@@ -76,6 +80,10 @@ def _load() -> ctypes.CDLL:
         _lib.oracle_argmax_f32.restype = None
         _lib.oracle_argmax_bf16.argtypes = [p, i64, i64, i64, p]
         _lib.oracle_argmax_bf16.restype = None
+        _lib.oracle_sample_f32.argtypes = [p, i64, i64, i64, f64, p, p]
+        _lib.oracle_sample_f32.restype = None
+        _lib.oracle_sample_bf16.argtypes = [p, i64, i64, i64, f64, p, p]
+        _lib.oracle_sample_bf16.restype = None
         _lib.oracle_accept_path.argtypes = [p, p, p, p, p, i64, i64, i64, p, p, p, p]
         _lib.oracle_accept_path.restype = ctypes.c_int
         _lib.oracle_kv_compact.argtypes = [
@@ -163,6 +171,24 @@ def argmax(logits, V: Optional[int] = None, bf16_bits: bool = False) -> np.ndarr
     else:
         x = _c(x, np.float32)
         _load().oracle_argmax_f32(_ptr(x), rows, V, x.shape[1], _ptr(out))
+    return out
+
+
+def sample(logits, temperature: float, u, V: Optional[int] = None, bf16_bits: bool = False) -> np.ndarray:
+    """One draw per row of a 2-D array (float32, or uint16 bf16 patterns) from
+    softmax(row / temperature), by inverse transform with the row's uniform
+    ``u[r]`` (float32); degenerate rows take their argmax."""
+    x = np.asarray(logits)
+    rows = x.shape[0]
+    V = x.shape[1] if V is None else int(V)
+    uu = _c(np.asarray(u, dtype=np.float32).reshape(rows), np.float32)
+    out = np.empty((rows,), dtype=np.int32)
+    if bf16_bits:
+        x = _c(x, np.uint16)
+        _load().oracle_sample_bf16(_ptr(x), rows, V, x.shape[1], float(temperature), _ptr(uu), _ptr(out))
+    else:
+        x = _c(x, np.float32)
+        _load().oracle_sample_f32(_ptr(x), rows, V, x.shape[1], float(temperature), _ptr(uu), _ptr(out))
     return out
 
 

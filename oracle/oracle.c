@@ -21,6 +21,11 @@
  *   - oracle_argmax_*       : the target's own greedy prediction per node,
  *                             temperature 0 (Sec. 2 "Speculative decoding";
  *                             Table 2, Temperature = 0), a linear scan.
+ *   - oracle_sample_*       : the target's own sample per node at temperature
+ *                             tau > 0 (Sec. 2 "Speculative decoding": each
+ *                             draft token is checked against the output of the
+ *                             target's own sampling; Table 2, Temperature = 1),
+ *                             by inverse transform of softmax(x / tau).
  *   - oracle_accept_path    : sequential acceptance -- drafts are accepted in
  *                             order while they equal the target's prediction,
  *                             and the target's own token replaces the first
@@ -47,7 +52,12 @@
  *     sibling tokens the matching path is unique); the root's own token is
  *     never checked; the accepted length counts the bonus (target) token;
  *   - at most max_path - 1 drafts are accepted (path and out_tokens rows hold
- *     max_path entries); entries past the accepted length are set to -1.
+ *     max_path entries); entries past the accepted length are set to -1;
+ *   - at temperature tau > 0 the target's own output at a node is one draw
+ *     from softmax(x / tau), taken by inverse transform with a uniform u that
+ *     the caller passes in: the smallest v whose cumulative weight exceeds
+ *     u times the total; acceptance then compares drafts with these draws
+ *     exactly as with the argmax at temperature 0.
  *
  * bf16 values are handled as their raw 16-bit patterns; widening bf16 to
  * double is exact.
@@ -247,6 +257,58 @@ void oracle_argmax_bf16(const uint16_t *logits, int64_t rows, int64_t V, int64_t
       if (argmax_better(bf16_bits_to_double(x[i]), bf16_bits_to_double(x[best]))) best = i;
     out[r] = (int32_t)best;
   }
+}
+
+/* One draw from softmax(x / tau) by inverse transform (x has V values):
+ *   M = max_v x_v,  w_v = exp((x_v - M) / tau),  Z = sum_v w_v,
+ *   draw = min { v : w_0 + ... + w_v > u * Z },
+ * with u clamped to [0, 1] (NaN counts as 0); when no v qualifies (u = 1), the
+ * last v with w_v > 0. A row holding a NaN, with maximum +inf, or with every
+ * value -inf has no such distribution: its draw is its argmax (the first NaN,
+ * else the first +inf, else index 0). */
+static int64_t sample_row(const double *x, int64_t V, double tau, double u) {
+  int64_t best = 0;
+  for (int64_t i = 1; i < V; ++i)
+    if (argmax_better(x[i], x[best])) best = i;
+  const double M = x[best];
+  if (isnan(M) || isinf(M)) return best;
+  if (!(u > 0.0)) u = 0.0;
+  if (u > 1.0) u = 1.0;
+  double Z = 0.0;
+  for (int64_t v = 0; v < V; ++v) Z += exp((x[v] - M) / tau);
+  const double target = u * Z;
+  double cum = 0.0;
+  int64_t last_pos = best;
+  for (int64_t v = 0; v < V; ++v) {
+    const double w = exp((x[v] - M) / tau);
+    cum += w;
+    if (w > 0.0) last_pos = v;
+    if (cum > target) return v;
+  }
+  return last_pos;
+}
+
+/* oracle_sample_f32: out[r] = one draw from softmax(logits[r, 0 .. V-1] / tau)
+ * with the uniform u[r] (see sample_row). */
+void oracle_sample_f32(const float *logits, int64_t rows, int64_t V, int64_t row_stride, double tau,
+                       const float *u, int32_t *out) {
+  double *x = (double *)malloc((size_t)V * sizeof(double));
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t v = 0; v < V; ++v) x[v] = (double)logits[r * row_stride + v];
+    out[r] = (int32_t)sample_row(x, V, tau, (double)u[r]);
+  }
+  free(x);
+}
+
+/* oracle_sample_bf16: the same over bf16 bit patterns widened to double. */
+void oracle_sample_bf16(const uint16_t *logits, int64_t rows, int64_t V, int64_t row_stride, double tau,
+                        const float *u, int32_t *out) {
+  double *x = (double *)malloc((size_t)V * sizeof(double));
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t v = 0; v < V; ++v) x[v] = bf16_bits_to_double(logits[r * row_stride + v]);
+    out[r] = (int32_t)sample_row(x, V, tau, (double)u[r]);
+  }
+  free(x);
 }
 
 /* Depth of node c (edges from the root); the tree is already checked. */
