@@ -211,6 +211,54 @@ dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int
                                    int32_t *status_word, dreams_stream_t stream);
 
 /*
+ * Temperature sampling: one draw per row from softmax(x / temperature), the
+ * target's own sample at temperature tau > 0 (Sec. 2 "Speculative decoding":
+ * each draft token is checked against the output of the target's own
+ * sampling; Table 2, Temperature = 1), by inverse transform with the row's
+ * uniform u_r = uniforms[r]:
+ *     M = max_v x_v,  w_v = exp((x_v - M) / tau),  Z = sum_v w_v
+ *     out_idx[r] = min { v : w_0 + ... + w_v > u_r Z }
+ * with u_r clamped to [0, 1] (NaN counts as 0); when no v qualifies (u_r = 1)
+ * the last v with w_v > 0. Rows holding a NaN, with maximum +inf, or with
+ * every value -inf take their argmax (the order of dreams_vocab_argmax).
+ * logits: f32 or bf16, rows x row_stride elements, row_stride >= V.
+ * uniforms: device f32 [rows] (the caller's random numbers). temperature:
+ * finite, > 0, with log2(e) / temperature finite in f32. The weights are f32
+ * (hardware exp2 of the scaled difference, subnormals flushed) summed in a
+ * fixed order per row, so a draw can differ from the exact-arithmetic draw
+ * only when u_r Z lies within rounding of a cumulative sum. Two launches:
+ * per-segment statistics (max and weight sum of every 256 values), then one
+ * warp per row that finds the segment and the value. The workspace holds
+ * 8 bytes per 256 values per row and no state between calls.
+ */
+size_t dreams_vocab_sample_workspace_size(int64_t rows, int64_t V);
+dreams_status_t dreams_vocab_sample(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
+                                    int64_t row_stride, float temperature, const float *uniforms,
+                                    int32_t *out_idx, void *workspace, size_t workspace_bytes,
+                                    dreams_stream_t stream);
+
+/*
+ * The verification tail at temperature tau > 0: the draw of
+ * dreams_vocab_sample for the rows of tree nodes (row b * T_max + i for
+ * i < tree_len[b], uniforms [B, T_max]) takes the place of the argmax, then
+ * dreams_accept_path and dreams_kv_compact run as in dreams_verify_step: a
+ * draft is accepted when it equals the target's draw at its parent, and the
+ * draw at the last accepted node is the bonus token (Sec. 2 "Speculative
+ * decoding"). sample_out ([B, T_max], may be NULL) receives the draws of the
+ * rows computed. Two kernel launches: the segment statistics, then (one CTA
+ * per sequence, chained by programmatic dependent launch) the draws, the walk
+ * and the compaction.
+ */
+size_t dreams_verify_step_sampled_workspace_size(const dreams_tree_t *tree, int64_t V);
+dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dtype, int64_t V,
+                                           int64_t row_stride, const dreams_tree_t *tree,
+                                           const dreams_kv_cache_t *kv, int32_t max_path, float temperature,
+                                           const float *uniforms, int32_t *sample_out, int32_t *accept_len,
+                                           int32_t *path, int32_t *out_tokens, int32_t *new_kv_len,
+                                           void *workspace, size_t workspace_bytes, int32_t *status_word,
+                                           dreams_stream_t stream);
+
+/*
  * Row-wise argmax for callers that cannot allocate device memory. The paper
  * has no counterpart to this call; it exists for integration. Some callers
  * cannot allocate, or cannot hand out a workspace, when the argmax runs: a

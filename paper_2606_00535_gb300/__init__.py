@@ -86,6 +86,11 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, p, p, p, p,
                                                           p, p, sz, p, p]),
                     "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
+                    "dreams_vocab_sample_workspace_size": (sz, [i64, i64]),
+                    "dreams_vocab_sample": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, f32, p, p, p, sz, p]),
+                    "dreams_verify_step_sampled_workspace_size": (sz, [ptr, i64]),
+                    "dreams_verify_step_sampled": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, f32, p,
+                                                                  p, p, p, p, p, p, sz, p, p]),
                     "dreams_status_string": (ctypes.c_char_p, [ctypes.c_int]),
                     "dreams_version": (i32, []),
                     "dreams_last_cuda_error": (i32, []),
@@ -295,6 +300,35 @@ def vocab_argmax_noalloc(logits: torch.Tensor, out: torch.Tensor, stream=None) -
     return out
 
 
+def vocab_sample(logits: torch.Tensor, temperature: float, uniforms: torch.Tensor,
+                 out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                 stream=None) -> torch.Tensor:
+    """One draw per row of a 2-D (or flattened leading dims) f32 / bf16 tensor
+    from softmax(row / temperature), by inverse transform with the row's
+    uniform (``uniforms``: f32, one per row, on the same device)."""
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    V = int(logits.shape[-1])
+    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
+    if x.stride(-1) != 1:
+        raise ValueError("logits rows must be contiguous")
+    rows = int(x.shape[0])
+    _need(uniforms, "uniforms", torch.float32, logits.device)
+    if uniforms.numel() != rows:
+        raise ValueError("uniforms must hold one value per row")
+    if out is None:
+        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=logits.device)
+    _need(out, "out", torch.int32, logits.device)
+    need = int(_lib().dreams_vocab_sample_workspace_size(rows, V))
+    if workspace is None:
+        workspace = _workspace("sample", need, logits.device, stream)
+    st = _lib().dreams_vocab_sample(
+        _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), float(temperature),
+        _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
+    _check("dreams_vocab_sample", st)
+    return out
+
+
 def _walk_outputs(B: int, max_path: int, dev):
     return (torch.empty(B, dtype=torch.int32, device=dev),
             torch.empty((B, max_path), dtype=torch.int32, device=dev),
@@ -326,6 +360,10 @@ def kv_compact(kv: KVCache, kv_len: torch.Tensor, accept_len: torch.Tensor, path
     _check("dreams_kv_compact", st)
 
 
+def verify_step_sampled_workspace_size(tree: Tree, V: int) -> int:
+    return int(_lib().dreams_verify_step_sampled_workspace_size(ctypes.byref(tree._c), V))
+
+
 def verify_step_workspace_size(tree: Tree, V: int) -> int:
     return int(_lib().dreams_verify_step_workspace_size(ctypes.byref(tree._c), V))
 
@@ -355,4 +393,36 @@ def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
         _ptr(toks), _ptr(nkl), _ptr(workspace), 0 if workspace is None else workspace.numel(), _ptr(status),
         _stream(stream))
     _check("dreams_verify_step", st)
+    return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
+
+
+def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int, temperature: float,
+                        uniforms: torch.Tensor, sample_out: Optional[torch.Tensor] = None,
+                        outputs: Optional[tuple] = None, workspace: Optional[torch.Tensor] = None,
+                        status: Optional[torch.Tensor] = None, stream=None) -> dict:
+    """The verification tail at temperature > 0: the target's draw per tree
+    node (``uniforms``: f32 [B, T_max]) takes the place of the argmax, then
+    acceptance and KV compaction, in one call (two kernel launches)."""
+    dev = tree.parent.device
+    if logits.dtype not in (torch.float32, torch.bfloat16) or logits.device != dev:
+        raise TypeError("logits must be float32/bfloat16 on the tree's device")
+    if logits.dim() != 3 or tuple(logits.shape[:2]) != (tree.B, tree.T_max) or logits.stride(-1) != 1 or \
+            logits.stride(0) != logits.shape[1] * logits.stride(1):
+        raise ValueError("logits must be [B, T_max, V] with uniformly strided contiguous rows")
+    _need(uniforms, "uniforms", torch.float32, dev)
+    if tuple(uniforms.shape) != (tree.B, tree.T_max):
+        raise ValueError("uniforms must be [B, T_max]")
+    V = int(logits.shape[2])
+    if sample_out is not None:
+        _need(sample_out, "sample_out", torch.int32, dev)
+    acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
+    need = verify_step_sampled_workspace_size(tree, V)
+    if workspace is None:
+        workspace = _workspace("step_sampled", need, dev, stream)
+    st = _lib().dreams_verify_step_sampled(
+        _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
+        ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature), _ptr(uniforms),
+        _ptr(sample_out), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(workspace),
+        0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
+    _check("dreams_verify_step_sampled", st)
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}

@@ -64,6 +64,12 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
   asm("max.NaN.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
   return d;
 }
+// 2^x by the hardware approximation (ex2.approx, subnormals flushed to zero).
+__device__ __forceinline__ float exp2f_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 template <typename T>
 struct Elem;
@@ -239,6 +245,283 @@ __global__ void __launch_bounds__(ARGMAX_THREADS) vocab_argmax_kernel(const Argm
   block_argmax<T>(base, begin, end, p.vec_ok, key, idx);
   if (row_combine(p.nchunk, p.slot + row, p.cnt + row, key, idx, row_idx) && threadIdx.x == 0)
     p.out[row] = row_idx;
+}
+
+
+// ------------------------------------------------------------------ temperature sampling
+// One draw per row from softmax(x / tau) by inverse transform with the row's
+// uniform u (the target's own sample, paper Sec. 2 "Speculative decoding";
+// Table 2, Temperature = 1). A row is cut into segments of SEG consecutive
+// values, one warp per segment, 8 values per lane.
+//   stage 1 (data-parallel over rows x segment ranges): per segment its
+//     maximum m (NaN-propagating) and s = sum of 2^((x - m) k), k = log2(e) /
+//     tau, each lane summing its 8 values in index order, then a xor-shuffle
+//     tree over the lanes;
+//   stage 2 (one warp per row): the row maximum M over the segments; Z = the
+//     segments' s scaled by 2^((m - M) k), summed in segment order (each lane
+//     a contiguous block, then an inclusive warp scan); the segment where the
+//     running sum first exceeds u Z; that segment re-read in index order and
+//     the value where the running sum crosses.
+// Where fp32 rounding leaves the crossing just past a segment's total, the
+// draw is the segment's last value of positive weight. Rows holding a NaN, with
+// maximum +inf, or with every value -inf take their argmax.
+constexpr int SEG = 256;
+constexpr int SAMPLE_THREADS = 256;  // stage 1: 8 warps, each one segment at a time
+
+struct SampleParams {
+  const void *logits;
+  int64_t V, row_stride;
+  int32_t nseg;         // segments per row
+  int32_t seg_per_cta;  // segments per stage-1 CTA
+  int32_t ncta_row;     // stage-1 CTAs per row
+  float k2;             // log2(e) / tau
+  bool vec_ok;          // rows start 16-byte aligned
+  const float *u;       // [rows]
+  float2 *seg;          // [rows][nseg] (m, s)
+};
+
+// The 8 values of this lane in segment g (elements g * SEG + 8 lane + i), as
+// floats; values at or past V read as -inf.
+template <typename T>
+__device__ __forceinline__ void seg_load(const T *row, int64_t V, bool vec_ok, int64_t g, float (&x)[8]) {
+  const int lane = threadIdx.x & 31;
+  const int64_t e0 = g * SEG + 8 * lane;
+  if (vec_ok && e0 + 8 <= V) {
+    if (sizeof(T) == 2) {
+      const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row + e0));
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+      }
+    } else {
+      const uint4 a = __ldcs(reinterpret_cast<const uint4 *>(row + e0));
+      const uint4 b = __ldcs(reinterpret_cast<const uint4 *>(row + e0) + 1);
+      x[0] = __uint_as_float(a.x), x[1] = __uint_as_float(a.y), x[2] = __uint_as_float(a.z);
+      x[3] = __uint_as_float(a.w), x[4] = __uint_as_float(b.x), x[5] = __uint_as_float(b.y);
+      x[6] = __uint_as_float(b.z), x[7] = __uint_as_float(b.w);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) x[i] = e0 + i < V ? __uint_as_float(Elem<T>::bits(row, e0 + i)) : -INFINITY;
+  }
+}
+
+// Lane sum of 2^((x - m) k) over its 8 values, in index order.
+__device__ __forceinline__ float seg_lane_sum(const float (&x)[8], float m, float k2) {
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) s += exp2f_approx((x[i] - m) * k2);
+  return s;
+}
+
+// Stage 1 for segments [g0, g1) of one row: warp w takes g0 + w, g0 + w + 8, ...
+template <typename T>
+__device__ void sample_stats(const SampleParams &p, const T *row, float2 *seg_row, int64_t g0, int64_t g1) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr int NW = SAMPLE_THREADS / 32;
+  int64_t g = g0 + warp;
+  for (; g + NW < g1; g += 2 * NW) {  // two segments in flight per warp
+    float xa[8], xb[8];
+    seg_load<T>(row, p.V, p.vec_ok, g, xa);
+    seg_load<T>(row, p.V, p.vec_ok, g + NW, xb);
+    float ma = xa[0], mb = xb[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) {
+      ma = fmax_nan(ma, xa[i]);
+      mb = fmax_nan(mb, xb[i]);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      ma = fmax_nan(ma, __shfl_xor_sync(0xffffffffu, ma, off));
+      mb = fmax_nan(mb, __shfl_xor_sync(0xffffffffu, mb, off));
+    }
+    float sa = seg_lane_sum(xa, ma, p.k2), sb = seg_lane_sum(xb, mb, p.k2);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      sa += __shfl_xor_sync(0xffffffffu, sa, off);
+      sb += __shfl_xor_sync(0xffffffffu, sb, off);
+    }
+    if (lane == 0) {
+      seg_row[g] = make_float2(ma, sa);
+      seg_row[g + NW] = make_float2(mb, sb);
+    }
+  }
+  for (; g < g1; g += NW) {
+    float x[8];
+    seg_load<T>(row, p.V, p.vec_ok, g, x);
+    float m = x[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) m = fmax_nan(m, x[i]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmax_nan(m, __shfl_xor_sync(0xffffffffu, m, off));
+    float s = seg_lane_sum(x, m, p.k2);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) seg_row[g] = make_float2(m, s);
+  }
+}
+
+// Stage 2 for one row (one warp): returns the draw. seg_row was written by
+// stage 1 (possibly by other CTAs of a completed grid: read through L2).
+template <typename T>
+__device__ int sample_select_warp(const SampleParams &p, const T *row, const float2 *seg_row, float u) {
+  const int lane = threadIdx.x & 31;
+  const int nseg = p.nseg;
+  const int q = (nseg + 31) / 32;
+  const int gb = min(nseg, lane * q), ge = min(nseg, gb + q);  // this lane's block of segments
+  float lm = -INFINITY;
+  for (int g = gb; g < ge; ++g) lm = fmax_nan(lm, __ldcg(seg_row + g).x);
+  float M = lm;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmax_nan(M, __shfl_xor_sync(0xffffffffu, M, off));
+  if (M == -INFINITY) return 0;  // every value -inf: the argmax is index 0
+  if (isnan(M) || M == INFINITY) {
+    // degenerate: the first NaN, else the first +inf (the argmax order)
+    int first = INT_MAX;
+    for (int g = gb; g < ge && first == INT_MAX; ++g) {
+      const float m = __ldcg(seg_row + g).x;
+      if (isnan(M) ? isnan(m) : m == INFINITY) first = g;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) first = min(first, __shfl_xor_sync(0xffffffffu, first, off));
+    if (first == INT_MAX) return 0;
+    float x[8];
+    seg_load<T>(row, p.V, false, first, x);
+    int hit = 8;
+#pragma unroll
+    for (int i = 7; i >= 0; --i)
+      if (isnan(M) ? isnan(x[i]) : x[i] == INFINITY) hit = i;
+    const unsigned bal = __ballot_sync(0xffffffffu, hit < 8);
+    const int l0 = __ffs(bal) - 1;
+    return first * SEG + 8 * l0 + __shfl_sync(0xffffffffu, hit, l0);
+  }
+  // weights of this lane's segments in the row's scale, their block sum, and
+  // an inclusive scan over the lanes (segment order)
+  float wsum = 0.f;
+  for (int g = gb; g < ge; ++g) {
+    const float2 ms = __ldcg(seg_row + g);
+    if (ms.x != -INFINITY) wsum += ms.y * exp2f_approx((ms.x - M) * p.k2);
+  }
+  float inc = wsum;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, inc, off);
+    if (lane >= off) inc += y;
+  }
+  const float Z = __shfl_sync(0xffffffffu, inc, 31);
+  const float uc = u > 0.f ? fminf(u, 1.f) : 0.f;  // NaN and negatives count as 0
+  const float t = uc * Z;
+  const unsigned cross = __ballot_sync(0xffffffffu, inc > t);
+  int gs = -1;         // segment holding the draw
+  float r = 0.f;       // what is left of t at the start of that segment, in its own scale
+  bool tail = false;   // no crossing: take the last value of positive weight
+  if (cross) {
+    const int L = __ffs(cross) - 1;
+    if (lane == L) {
+      float acc = inc - wsum;
+      int last = -1;
+      float last_r = 0.f;
+      for (int g = gb; g < ge; ++g) {
+        const float2 ms = __ldcg(seg_row + g);
+        if (ms.x == -INFINITY) continue;
+        const float sc = exp2f_approx((ms.x - M) * p.k2);
+        const float c = ms.y * sc;
+        if (c > 0.f) {
+          last = g;
+          last_r = fmaxf(t - acc, 0.f) / sc;
+        }
+        if (acc + c > t) {
+          gs = g;
+          r = fmaxf(t - acc, 0.f) / sc;  // >= 0: the draw has positive weight
+          break;
+        }
+        acc += c;
+      }
+      if (gs < 0) {
+        gs = last;
+        r = last_r;
+        tail = true;
+      }
+    }
+    gs = __shfl_sync(0xffffffffu, gs, L);
+    r = __shfl_sync(0xffffffffu, r, L);
+    tail = __shfl_sync(0xffffffffu, tail, L);
+  } else {
+    // t >= Z (u = 1, or rounding): the last segment of positive weight
+    int last = -1;
+    for (int g = gb; g < ge; ++g) {
+      const float2 ms = __ldcg(seg_row + g);
+      if (ms.x != -INFINITY && ms.y * exp2f_approx((ms.x - M) * p.k2) > 0.f) last = g;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, off));
+    gs = last;
+    tail = true;
+  }
+  if (gs < 0) return 0;
+  // the segment again, in index order, in its own scale
+  const float m = __ldcg(seg_row + gs).x;
+  float x[8];
+  seg_load<T>(row, p.V, p.vec_ok, gs, x);
+  float w[8], ls = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    w[i] = exp2f_approx((x[i] - m) * p.k2);
+    ls += w[i];
+  }
+  float linc = ls;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, linc, off);
+    if (lane >= off) linc += y;
+  }
+  int pick = -1;
+  const unsigned lc = tail ? 0u : __ballot_sync(0xffffffffu, linc > r);
+  if (lc) {
+    const int L = __ffs(lc) - 1;
+    if (lane == L) {
+      float acc = linc - ls;
+      for (int i = 0; i < 8; ++i) {
+        acc += w[i];
+        if (w[i] > 0.f) pick = i;
+        if (acc > r) {
+          pick = i;
+          break;
+        }
+      }
+    }
+    pick = __shfl_sync(0xffffffffu, pick, L);
+    return gs * SEG + 8 * (__ffs(lc) - 1) + pick;
+  }
+  // the segment's last value of positive weight
+  int li = -1;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    if (w[i] > 0.f) li = i;
+  const unsigned has = __ballot_sync(0xffffffffu, li >= 0);
+  if (!has) return gs * SEG;
+  const int L = 31 - __clz(has);
+  return gs * SEG + 8 * L + __shfl_sync(0xffffffffu, li, L);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(SAMPLE_THREADS) vocab_sample_stats_kernel(const SampleParams p) {
+  const int64_t row = blockIdx.x / p.ncta_row;
+  const int c = blockIdx.x % p.ncta_row;
+  const T *base = static_cast<const T *>(p.logits) + row * p.row_stride;
+  const int64_t g0 = int64_t(c) * p.seg_per_cta, g1 = std::min<int64_t>(p.nseg, g0 + p.seg_per_cta);
+  sample_stats<T>(p, base, p.seg + row * p.nseg, g0, g1);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) vocab_sample_select_kernel(const SampleParams p, int64_t rows, int32_t *out) {
+  const int64_t row = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  const T *base = static_cast<const T *>(p.logits) + row * p.row_stride;
+  const int idx = sample_select_warp<T>(p, base, p.seg + row * p.nseg, __ldg(p.u + row));
+  if ((threadIdx.x & 31) == 0) out[row] = idx;
 }
 
 // ------------------------------------------------------------------ tree walk
@@ -489,6 +772,8 @@ __global__ void __launch_bounds__(TAIL_THREADS) kv_compact_kernel(const KVParams
 
 struct StepParams {
   ArgmaxParams am;
+  SampleParams sp;
+  bool sampled;  // predictions are draws at temperature tau (sp), not argmaxes (am)
   TreeParams tr;
   KVParams kv;
   int32_t max_path;
@@ -520,9 +805,28 @@ __global__ void __launch_bounds__(ARGMAX_THREADS) verify_rows_kernel(const StepP
     p.pred[rb + i] = row_idx;
 }
 
+// Launch 1 of the sampled verification tail. grid.x = B * T_max * ncta_row:
+// (sequence, tree node, segment range); padding nodes return at once. Stage 1
+// of the draw (segment statistics) of the node's row.
+template <typename T>
+__global__ void __launch_bounds__(SAMPLE_THREADS) verify_sample_rows_kernel(const StepParams p) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int ncta = p.sp.ncta_row;
+  const int c = blockIdx.x % ncta;
+  const int rowg = blockIdx.x / ncta;
+  const int b = rowg / p.tr.T_max, i = rowg % p.tr.T_max;
+  const int tl = __ldg(p.tr.tree_len + b);
+  if (tl < 1 || tl > p.tr.T_max || i >= tl) return;
+  const int64_t r = int64_t(b) * p.tr.T_max + i;
+  const T *row = static_cast<const T *>(p.sp.logits) + r * p.sp.row_stride;
+  const int64_t g0 = int64_t(c) * p.sp.seg_per_cta, g1 = std::min<int64_t>(p.sp.nseg, g0 + p.sp.seg_per_cta);
+  sample_stats<T>(p.sp, row, p.sp.seg + r * p.sp.nseg, g0, g1);
+}
+
 // Launch 2 of the verification tail, one CTA per sequence, chained to launch 1
 // by programmatic dependent launch (it may start early and waits until launch
 // 1 has completed): the acceptance walk, its outputs, and the KV compaction.
+template <typename LT>
 __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepParams p) {
   __shared__ int32_t s_path[65];
   __shared__ int64_t s_src[65], s_dst[65];
@@ -532,6 +836,16 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
   const int64_t rb = int64_t(b) * Tm;
   const int T = __ldg(p.tr.tree_len + b);
   const int L = __ldg(p.tr.kv_len + b);
+  if (p.sampled && T >= 1 && T <= Tm) {
+    // stage 2 of the draws: one warp per node row
+    for (int i = threadIdx.x >> 5; i < T; i += TAIL_THREADS / 32) {
+      const int64_t r = rb + i;
+      const LT *row = static_cast<const LT *>(p.sp.logits) + r * p.sp.row_stride;
+      const int idx = sample_select_warp<LT>(p.sp, row, p.sp.seg + r * p.sp.nseg, __ldg(p.sp.u + r));
+      if ((threadIdx.x & 31) == 0) p.pred[r] = idx;
+    }
+    __syncthreads();
+  }
   if (threadIdx.x < 32) {
     WalkOut w{-1, 0};
     if (T < 1 || T > Tm) w.bad = DREAMS_DATA_BAD_TREE_LEN;
@@ -576,6 +890,43 @@ ArgmaxPlan plan_argmax(int64_t rows, int64_t V) {
 }
 
 size_t argmax_ws(int64_t rows) { return align_up(size_t(rows) * 8, 256) + align_up(size_t(rows) * 4, 256); }
+
+struct SamplePlan {
+  int32_t nseg, seg_per_cta, ncta_row;
+};
+
+SamplePlan plan_sample(int64_t rows, int64_t V) {
+  // about four stage-1 CTAs per SM across the grid, >= 8 segments per CTA
+  const int64_t nseg = (V + SEG - 1) / SEG;
+  const int64_t target = int64_t(num_sms()) * 4;
+  int64_t ncta = (target + rows - 1) / std::max<int64_t>(rows, 1);
+  ncta = std::max<int64_t>(1, std::min<int64_t>(ncta, (nseg + 7) / 8));
+  const int64_t per = (nseg + ncta - 1) / ncta;
+  return {int32_t(nseg), int32_t(per), int32_t((nseg + per - 1) / per)};
+}
+
+size_t sample_ws(int64_t rows, int64_t V) { return align_up(size_t(rows) * size_t((V + SEG - 1) / SEG) * 8, 256); }
+
+// Checks and fills the sampling parameters shared by both entry points.
+bool sample_params(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V, int64_t row_stride,
+                   float temperature, const float *uniforms, void *seg_ws, SampleParams &p, int64_t &ctas) {
+  const float k2 = 1.4426950408889634f / temperature;
+  if (!(temperature > 0.f) || !isfinite(temperature) || !isfinite(k2) || uniforms == nullptr) return false;
+  const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
+  const SamplePlan pl = plan_sample(rows, V);
+  p.logits = logits;
+  p.V = V;
+  p.row_stride = row_stride;
+  p.nseg = pl.nseg;
+  p.seg_per_cta = pl.seg_per_cta;
+  p.ncta_row = pl.ncta_row;
+  p.k2 = k2;
+  p.vec_ok = aligned16(logits) && (row_stride * int64_t(esz)) % 16 == 0;
+  p.u = uniforms;
+  p.seg = static_cast<float2 *>(seg_ws);
+  ctas = rows * pl.ncta_row;
+  return true;
+}
 
 bool kv_params(const dreams_kv_cache_t *kv, KVParams &out) {
   if (kv == nullptr || kv->k == nullptr || kv->v == nullptr || kv->n_layers < 1 || kv->Hkv < 1 ||
@@ -733,7 +1084,104 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_tail_kernel, p);
+  const cudaError_t e = dtype == DREAMS_F32 ? cudaLaunchKernelEx(&cfg, verify_tail_kernel<float>, p)
+                                             : cudaLaunchKernelEx(&cfg, verify_tail_kernel<__nv_bfloat16>, p);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
+  return check_launch();
+}
+
+extern "C" size_t dreams_vocab_sample_workspace_size(int64_t rows, int64_t V) {
+  if (rows < 1 || V < 1) return 0;
+  return sample_ws(rows, V);
+}
+
+extern "C" dreams_status_t dreams_vocab_sample(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
+                                               int64_t row_stride, float temperature, const float *uniforms,
+                                               int32_t *out_idx, void *workspace, size_t workspace_bytes,
+                                               dreams_stream_t stream) {
+  if (logits == nullptr || out_idx == nullptr || rows < 1 || V < 1 || V > INT_MAX - SEG || row_stride < V)
+    return DREAMS_ERR_INVALID_ARG;
+  if (dtype != DREAMS_F32 && dtype != DREAMS_BF16) return DREAMS_ERR_UNSUPPORTED;
+  const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
+  if (reinterpret_cast<uintptr_t>(logits) % esz || (reinterpret_cast<uintptr_t>(uniforms) & 3))
+    return DREAMS_ERR_INVALID_ARG;
+  if (workspace == nullptr || workspace_bytes < sample_ws(rows, V) || !aligned16(workspace))
+    return DREAMS_ERR_WORKSPACE;
+  SampleParams p{};
+  int64_t ctas = 0;
+  if (!sample_params(logits, dtype, rows, V, row_stride, temperature, uniforms, workspace, p, ctas))
+    return DREAMS_ERR_INVALID_ARG;
+  if (ctas > INT_MAX || (rows + 7) / 8 > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const dim3 g1(static_cast<unsigned>(ctas)), g2(static_cast<unsigned>((rows + 7) / 8));
+  if (dtype == DREAMS_F32) {
+    vocab_sample_stats_kernel<float><<<g1, SAMPLE_THREADS, 0, s>>>(p);
+    vocab_sample_select_kernel<float><<<g2, 256, 0, s>>>(p, rows, out_idx);
+  } else {
+    vocab_sample_stats_kernel<__nv_bfloat16><<<g1, SAMPLE_THREADS, 0, s>>>(p);
+    vocab_sample_select_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(p, rows, out_idx);
+  }
+  return check_launch();
+}
+
+extern "C" size_t dreams_verify_step_sampled_workspace_size(const dreams_tree_t *tree, int64_t V) {
+  if (tree == nullptr || tree->B < 1 || tree->T_max < 1 || V < 1) return 0;
+  const int64_t rows = int64_t(tree->B) * tree->T_max;
+  return sample_ws(rows, V) + align_up(size_t(rows) * 4, 256);
+}
+
+extern "C" dreams_status_t dreams_verify_step_sampled(
+    const void *logits, dreams_dtype_t dtype, int64_t V, int64_t row_stride, const dreams_tree_t *tree,
+    const dreams_kv_cache_t *kv, int32_t max_path, float temperature, const float *uniforms, int32_t *sample_out,
+    int32_t *accept_len, int32_t *path, int32_t *out_tokens, int32_t *new_kv_len, void *workspace,
+    size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream) {
+  StepParams p{};
+  if (logits == nullptr || V < 1 || V > INT_MAX - SEG || row_stride < V || !tree_params(tree, true, p.tr) ||
+      !kv_params(kv, p.kv) || max_path < 1 || max_path > 65 || accept_len == nullptr || path == nullptr ||
+      out_tokens == nullptr || new_kv_len == nullptr)
+    return DREAMS_ERR_INVALID_ARG;
+  if (dtype != DREAMS_F32 && dtype != DREAMS_BF16) return DREAMS_ERR_UNSUPPORTED;
+  const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
+  if (reinterpret_cast<uintptr_t>(logits) % esz || (reinterpret_cast<uintptr_t>(uniforms) & 3))
+    return DREAMS_ERR_INVALID_ARG;
+  const int64_t rows = int64_t(tree->B) * tree->T_max;
+  const size_t need = dreams_verify_step_sampled_workspace_size(tree, V);
+  if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace)) return DREAMS_ERR_WORKSPACE;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  int64_t ctas = 0;
+  if (!sample_params(logits, dtype, rows, V, row_stride, temperature, uniforms, ws, p.sp, ctas))
+    return DREAMS_ERR_INVALID_ARG;
+  if (ctas > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  p.sampled = true;
+  int32_t *ws_pred = reinterpret_cast<int32_t *>(ws + sample_ws(rows, V));
+  p.pred = sample_out != nullptr ? sample_out : ws_pred;
+  p.pred_in_ws = false;
+  p.max_path = max_path;
+  p.accept_len = accept_len;
+  p.path = path;
+  p.out_tokens = out_tokens;
+  p.new_kv_len = new_kv_len;
+  p.status = status_word;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const dim3 grid(static_cast<unsigned>(ctas));
+  if (dtype == DREAMS_F32) verify_sample_rows_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  else verify_sample_rows_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  dreams_status_t st = check_launch();
+  if (st != DREAMS_OK) return st;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(tree->B));
+  cfg.blockDim = dim3(TAIL_THREADS);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = dtype == DREAMS_F32 ? cudaLaunchKernelEx(&cfg, verify_tail_kernel<float>, p)
+                                             : cudaLaunchKernelEx(&cfg, verify_tail_kernel<__nv_bfloat16>, p);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return DREAMS_ERR_CUDA;
