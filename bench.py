@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--config", default="batched", choices=[s.name for s in W.SPECS])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-sampled", action="store_true",
+                    help="skip the extra timing of the temperature-1 verification tail")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
     ap.add_argument("--load-seconds", type=float, default=1.0,
                     help="untimed steps run while the clock sampler starts (0 under a profiler)")
@@ -313,6 +315,35 @@ def run_dreams(args, rank, world, local):
         e2e_us = s0.elapsed_time(s1) / Ke * 1000.0
         e2e = {"value": round(e2e_us, 2), "unit": "us", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
+    # ---- the verification tail at temperature 1 (draws instead of argmaxes),
+    # timed apart from the headline step: same rotating inputs, CUDA events
+    sampled = None
+    if not args.no_sampled:
+        u = torch.rand((w.B, w.T_max), generator=torch.Generator().manual_seed(7)).to(dev)
+        ws_s = torch.zeros(dreams.verify_step_sampled_workspace_size(copies[0]["tree"], w.V), dtype=torch.uint8,
+                           device=dev)
+
+        def sampled_call(c):
+            dreams.verify_step_sampled(c["logits"], c["tree"], c["kv"], max_path, 1.0, u, outputs=c["outs"],
+                                       workspace=ws_s, status=status)
+
+        for i in range(4):
+            sampled_call(copies[i % 2])
+        Ks = max(3, min(K, 100))
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        s0.record(stream)
+        for i in range(Ks):
+            sampled_call(copies[i % 2])
+        s1.record(stream)
+        barrier()
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item()):#x} on valid input (sampled step)")
+        sampled_us = s0.elapsed_time(s1) / Ks * 1000.0
+        sampled = {"us": round(sampled_us, 2), "temperature": 1.0, "launches": dreams.VERIFY_STEP_SAMPLED_LAUNCHES,
+                   "launch": "eager", "GBps": round(argmax_bytes(w) / (sampled_us * 1e-6) / 1e9, 1)}
+
     ab, gb = attn_bytes(w), argmax_bytes(w)
     attn_avg_ms = sum(attn_ms) / K
     tail_avg_ms = sum(tail_ms) / K
@@ -334,6 +365,9 @@ def run_dreams(args, rank, world, local):
         "verify_step": {"us": round(tail_avg_ms * 1000, 2), "argmax_bytes": gb, "GBps": round(tail_gbs, 1),
                         "frac_measured_hbm": round(tail_gbs / peak, 4)},
     }
+    if sampled is not None:
+        sampled["frac_measured_hbm"] = round(sampled["GBps"] / peak, 4)
+        kernels["verify_step_sampled"] = sampled
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -226,10 +226,11 @@ dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t dtype, int
  * finite, > 0, with log2(e) / temperature finite in f32. The weights are f32
  * (hardware exp2 of the scaled difference, subnormals flushed) summed in a
  * fixed order per row, so a draw can differ from the exact-arithmetic draw
- * only when u_r Z lies within rounding of a cumulative sum. Two launches:
- * per-segment statistics (max and weight sum of every 256 values), then one
- * warp per row that finds the segment and the value. The workspace holds
- * 8 bytes per 256 values per row and no state between calls.
+ * only when u_r Z lies within rounding of a cumulative sum. Two launches,
+ * chained by programmatic dependent launch: CTAs over (row, range of
+ * 1024-value segments) store each segment's maximum and weight sum in the
+ * workspace (8 bytes per 1024 values per row); then one warp per row finds
+ * the segment and the value. The workspace holds no state between calls.
  */
 size_t dreams_vocab_sample_workspace_size(int64_t rows, int64_t V);
 dreams_status_t dreams_vocab_sample(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
@@ -245,9 +246,10 @@ dreams_status_t dreams_vocab_sample(const void *logits, dreams_dtype_t dtype, in
  * draft is accepted when it equals the target's draw at its parent, and the
  * draw at the last accepted node is the bonus token (Sec. 2 "Speculative
  * decoding"). sample_out ([B, T_max], may be NULL) receives the draws of the
- * rows computed. Two kernel launches: the segment statistics, then (one CTA
- * per sequence, chained by programmatic dependent launch) the draws, the walk
- * and the compaction.
+ * rows computed. Three kernel launches, chained by programmatic dependent
+ * launch: the two stages of the draws over the node rows, then the walk and
+ * the compaction (one CTA per sequence). The workspace holds no state between
+ * calls.
  */
 size_t dreams_verify_step_sampled_workspace_size(const dreams_tree_t *tree, int64_t V);
 dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dtype, int64_t V,

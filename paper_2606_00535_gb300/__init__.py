@@ -228,7 +228,8 @@ def tree_verify_attn_launches(kv: KVCache, tree: Tree, Hq: int) -> int:
     return int(_lib().dreams_tree_verify_attn_launches(ctypes.byref(kv._c), ctypes.byref(tree._c), Hq))
 
 
-VERIFY_STEP_LAUNCHES = 2  # dreams_verify_step: the argmax, then the walk and compaction
+VERIFY_STEP_LAUNCHES = 2
+VERIFY_STEP_SAMPLED_LAUNCHES = 3  # draw statistics, draw selection, walk + compaction  # dreams_verify_step: the argmax, then the walk and compaction
 
 
 def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, layer: int = 0,

@@ -251,41 +251,44 @@ __global__ void __launch_bounds__(ARGMAX_THREADS) vocab_argmax_kernel(const Argm
 // ------------------------------------------------------------------ temperature sampling
 // One draw per row from softmax(x / tau) by inverse transform with the row's
 // uniform u (the target's own sample, paper Sec. 2 "Speculative decoding";
-// Table 2, Temperature = 1). A row is cut into segments of SEG consecutive
-// values, one warp per segment, 8 values per lane.
+// Table 2, Temperature = 1). A row is cut into segments of SEG = 1024
+// consecutive values, one warp per segment; a segment is four steps of SUB =
+// 256 values, 8 consecutive values per lane in each step.
 //   stage 1 (data-parallel over rows x segment ranges): per segment its
 //     maximum m (NaN-propagating) and s = sum of 2^((x - m) k), k = log2(e) /
-//     tau, each lane summing its 8 values in index order, then a xor-shuffle
-//     tree over the lanes;
-//   stage 2 (one warp per row): the row maximum M over the segments; Z = the
-//     segments' s scaled by 2^((m - M) k), summed in segment order (each lane
-//     a contiguous block, then an inclusive warp scan); the segment where the
-//     running sum first exceeds u Z; that segment re-read in index order and
-//     the value where the running sum crosses.
+//     tau (lane sums, then a xor-shuffle tree);
+//   stage 2 (a second launch, one warp per row): the row maximum M and the
+//     total Z over the segments; the segment where the running sum, in
+//     segment order, first exceeds u Z; that segment re-read step by step in
+//     index order and the value where the running sum crosses.
+// Stage 1 keeps each lane's values as raw 16-byte words (the maximum of bf16
+// data by packed max instructions) so that it needs few registers and many
+// CTAs stream at once.
 // Where fp32 rounding leaves the crossing just past a segment's total, the
-// draw is the segment's last value of positive weight. Rows holding a NaN, with
-// maximum +inf, or with every value -inf take their argmax.
-constexpr int SEG = 256;
+// draw is the last value of positive weight before it. Rows holding a NaN,
+// with maximum +inf, or with every value -inf take their argmax.
+constexpr int SUB = 256;
+constexpr int SEG = 4 * SUB;
 constexpr int SAMPLE_THREADS = 256;  // stage 1: 8 warps, each one segment at a time
 
 struct SampleParams {
   const void *logits;
   int64_t V, row_stride;
   int32_t nseg;         // segments per row
-  int32_t seg_per_cta;  // segments per stage-1 CTA
-  int32_t ncta_row;     // stage-1 CTAs per row
+  int32_t seg_per_cta;  // segments per CTA
+  int32_t ncta_row;     // CTAs per row
   float k2;             // log2(e) / tau
   bool vec_ok;          // rows start 16-byte aligned
   const float *u;       // [rows]
   float2 *seg;          // [rows][nseg] (m, s)
 };
 
-// The 8 values of this lane in segment g (elements g * SEG + 8 lane + i), as
-// floats; values at or past V read as -inf.
+// The 8 values of this lane in step j of the row (elements j * SUB + 8 lane +
+// i), as floats; values at or past V read as -inf.
 template <typename T>
-__device__ __forceinline__ void seg_load(const T *row, int64_t V, bool vec_ok, int64_t g, float (&x)[8]) {
+__device__ __forceinline__ void sub_load(const T *row, int64_t V, bool vec_ok, int64_t j, float (&x)[8]) {
   const int lane = threadIdx.x & 31;
-  const int64_t e0 = g * SEG + 8 * lane;
+  const int64_t e0 = j * SUB + 8 * lane;
   if (vec_ok && e0 + 8 <= V) {
     if (sizeof(T) == 2) {
       const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row + e0));
@@ -308,220 +311,327 @@ __device__ __forceinline__ void seg_load(const T *row, int64_t V, bool vec_ok, i
   }
 }
 
-// Lane sum of 2^((x - m) k) over its 8 values, in index order.
-__device__ __forceinline__ float seg_lane_sum(const float (&x)[8], float m, float k2) {
-  float s = 0.f;
+// Raw 16-byte words of this lane in step j of the row (elements j * SUB + 8
+// lane + i): one word of 8 bf16 values, or two of 4 f32 values; values at or
+// past V read as -inf.
+template <typename T>
+__device__ __forceinline__ void sub_words(const T *row, int64_t V, bool vec_ok, int64_t j, uint4 (&w)[sizeof(T) / 2]) {
+  const int lane = threadIdx.x & 31;
+  const int64_t e0 = j * SUB + 8 * lane;
+  if (vec_ok && e0 + 8 <= V) {
 #pragma unroll
-  for (int i = 0; i < 8; ++i) s += exp2f_approx((x[i] - m) * k2);
+    for (int q = 0; q < int(sizeof(T)) / 2; ++q) w[q] = __ldcs(reinterpret_cast<const uint4 *>(row + e0) + q);
+  } else {
+    uint32_t b[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) b[i] = e0 + i < V ? Elem<T>::bits(row, e0 + i) : 0xff800000u;  // -inf
+    if (sizeof(T) == 2) {
+      w[0] = make_uint4((b[0] >> 16) | (b[1] & 0xffff0000u), (b[2] >> 16) | (b[3] & 0xffff0000u),
+                        (b[4] >> 16) | (b[5] & 0xffff0000u), (b[6] >> 16) | (b[7] & 0xffff0000u));
+    } else {
+#pragma unroll
+      for (int q = 0; q < int(sizeof(T)) / 2; ++q) w[q] = make_uint4(b[4 * q], b[4 * q + 1], b[4 * q + 2], b[4 * q + 3]);
+    }
+  }
+}
+
+// Maximum (NaN-propagating) and the sum of 2^((x - m) k) of raw words.
+__device__ __forceinline__ float words_max(const uint4 *w, int n, bool bf16) {
+  if (bf16) {
+    uint32_t a = bmax2_nan(bmax2_nan(w[0].x, w[0].y), bmax2_nan(w[0].z, w[0].w));
+    for (int q = 1; q < n; ++q) a = bmax2_nan(a, bmax2_nan(bmax2_nan(w[q].x, w[q].y), bmax2_nan(w[q].z, w[q].w)));
+    a = bmax2_nan(a, __byte_perm(a, 0, 0x1032));
+    return __uint_as_float(a << 16);
+  }
+  float m = fmax_nan(fmax_nan(__uint_as_float(w[0].x), __uint_as_float(w[0].y)),
+                     fmax_nan(__uint_as_float(w[0].z), __uint_as_float(w[0].w)));
+  for (int q = 1; q < n; ++q)
+    m = fmax_nan(m, fmax_nan(fmax_nan(__uint_as_float(w[q].x), __uint_as_float(w[q].y)),
+                             fmax_nan(__uint_as_float(w[q].z), __uint_as_float(w[q].w))));
+  return m;
+}
+__device__ __forceinline__ float words_sum(const uint4 *w, int n, bool bf16, float m, float k2) {
+  float s = 0.f;
+  for (int q = 0; q < n; ++q) {
+    const uint32_t v[4] = {w[q].x, w[q].y, w[q].z, w[q].w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (bf16) {
+        s += exp2f_approx((__uint_as_float(v[i] << 16) - m) * k2);
+        s += exp2f_approx((__uint_as_float(v[i] & 0xffff0000u) - m) * k2);
+      } else {
+        s += exp2f_approx((__uint_as_float(v[i]) - m) * k2);
+      }
+    }
+  }
   return s;
 }
 
-// Stage 1 for segments [g0, g1) of one row: warp w takes g0 + w, g0 + w + 8, ...
+// Stage 1 for segments [g0, g1) of one row: warp w takes g0 + w, g0 + w + 8,
+// ..., one segment (4 or 8 words per lane) at a time.
 template <typename T>
 __device__ void sample_stats(const SampleParams &p, const T *row, float2 *seg_row, int64_t g0, int64_t g1) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   constexpr int NW = SAMPLE_THREADS / 32;
-  int64_t g = g0 + warp;
-  for (; g + NW < g1; g += 2 * NW) {  // two segments in flight per warp
-    float xa[8], xb[8];
-    seg_load<T>(row, p.V, p.vec_ok, g, xa);
-    seg_load<T>(row, p.V, p.vec_ok, g + NW, xb);
-    float ma = xa[0], mb = xb[0];
+  constexpr int WPS = 4 * (int(sizeof(T)) / 2);  // words per lane per segment
+  constexpr int SPI = 1;                         // segments per iteration
+  constexpr bool BF = sizeof(T) == 2;
+  for (int64_t g = g0 + warp; g < g1; g += SPI * NW) {
+    uint4 w[SPI][WPS];
 #pragma unroll
-    for (int i = 1; i < 8; ++i) {
-      ma = fmax_nan(ma, xa[i]);
-      mb = fmax_nan(mb, xb[i]);
-    }
+    for (int k = 0; k < SPI; ++k) {
+      const int64_t gk = g + k * NW;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      ma = fmax_nan(ma, __shfl_xor_sync(0xffffffffu, ma, off));
-      mb = fmax_nan(mb, __shfl_xor_sync(0xffffffffu, mb, off));
-    }
-    float sa = seg_lane_sum(xa, ma, p.k2), sb = seg_lane_sum(xb, mb, p.k2);
+      for (int j = 0; j < 4; ++j) {
+        uint4(&wj)[sizeof(T) / 2] = *reinterpret_cast<uint4(*)[sizeof(T) / 2]>(&w[k][j * (sizeof(T) / 2)]);
+        if (gk < g1) sub_words<T>(row, p.V, p.vec_ok, 4 * gk + j, wj);
+        else
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      sa += __shfl_xor_sync(0xffffffffu, sa, off);
-      sb += __shfl_xor_sync(0xffffffffu, sb, off);
+          for (int q = 0; q < int(sizeof(T)) / 2; ++q) {
+            const uint32_t ninf = BF ? 0xff80ff80u : 0xff800000u;  // -inf
+            wj[q] = make_uint4(ninf, ninf, ninf, ninf);
+          }
+      }
     }
+    float m[SPI], sum[SPI];
+#pragma unroll
+    for (int k = 0; k < SPI; ++k) m[k] = words_max(w[k], WPS, BF);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+      for (int k = 0; k < SPI; ++k) m[k] = fmax_nan(m[k], __shfl_xor_sync(0xffffffffu, m[k], off));
+#pragma unroll
+    for (int k = 0; k < SPI; ++k) sum[k] = words_sum(w[k], WPS, BF, m[k], p.k2);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+      for (int k = 0; k < SPI; ++k) sum[k] += __shfl_xor_sync(0xffffffffu, sum[k], off);
     if (lane == 0) {
-      seg_row[g] = make_float2(ma, sa);
-      seg_row[g + NW] = make_float2(mb, sb);
+#pragma unroll
+      for (int k = 0; k < SPI; ++k)
+        if (g + k * NW < g1) seg_row[g + k * NW] = make_float2(m[k], sum[k]);
     }
-  }
-  for (; g < g1; g += NW) {
-    float x[8];
-    seg_load<T>(row, p.V, p.vec_ok, g, x);
-    float m = x[0];
-#pragma unroll
-    for (int i = 1; i < 8; ++i) m = fmax_nan(m, x[i]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) m = fmax_nan(m, __shfl_xor_sync(0xffffffffu, m, off));
-    float s = seg_lane_sum(x, m, p.k2);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    if (lane == 0) seg_row[g] = make_float2(m, s);
   }
 }
 
+// The 8 segment statistics of this lane in batch `base` (segments base + 8 lane
+// .. base + 8 lane + 7), loaded together; past nseg: (-inf, 0).
+__device__ __forceinline__ void seg_batch(const float2 *seg_row, int nseg, int base, float2 (&v)[8]) {
+  const int g0 = base + 8 * (threadIdx.x & 31);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = g0 + i < nseg ? __ldcg(seg_row + g0 + i) : make_float2(-INFINITY, 0.f);
+}
+
 // Stage 2 for one row (one warp): returns the draw. seg_row was written by
-// stage 1 (possibly by other CTAs of a completed grid: read through L2).
+// stage 1 (by other CTAs too: read through L2). The statistics are read in
+// batches of 256 segments, 8 consecutive ones per lane: one pass for the row
+// maximum M, the total Z (online rescaling per lane, then a shuffle tree) and
+// the first NaN or +inf segment; one pass for the running sums in segment
+// order (an inclusive warp scan per batch plus the carry of earlier batches)
+// up to the crossing; then the crossing segment's values.
 template <typename T>
 __device__ int sample_select_warp(const SampleParams &p, const T *row, const float2 *seg_row, float u) {
   const int lane = threadIdx.x & 31;
   const int nseg = p.nseg;
-  const int q = (nseg + 31) / 32;
-  const int gb = min(nseg, lane * q), ge = min(nseg, gb + q);  // this lane's block of segments
-  float lm = -INFINITY;
-  for (int g = gb; g < ge; ++g) lm = fmax_nan(lm, __ldcg(seg_row + g).x);
-  float M = lm;
+  const float k2 = p.k2;
+  // ---- pass 1: M, Z, and the first segment whose maximum is NaN / +inf
+  float m_l = -INFINITY, z_l = 0.f;
+  int first_nan = INT_MAX, first_inf = INT_MAX;
+  for (int base = 0; base < nseg; base += 256) {
+    float2 v[8];
+    seg_batch(seg_row, nseg, base, v);
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) M = fmax_nan(M, __shfl_xor_sync(0xffffffffu, M, off));
-  if (M == -INFINITY) return 0;  // every value -inf: the argmax is index 0
-  if (isnan(M) || M == INFINITY) {
-    // degenerate: the first NaN, else the first +inf (the argmax order)
-    int first = INT_MAX;
-    for (int g = gb; g < ge && first == INT_MAX; ++g) {
-      const float m = __ldcg(seg_row + g).x;
-      if (isnan(M) ? isnan(m) : m == INFINITY) first = g;
+    for (int i = 0; i < 8; ++i) {
+      const int g = base + 8 * lane + i;
+      if (isnan(v[i].x)) {
+        first_nan = min(first_nan, g);
+      } else if (v[i].x == INFINITY) {
+        first_inf = min(first_inf, g);
+      } else if (v[i].x != -INFINITY) {
+        if (v[i].x > m_l) {
+          z_l = (m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - v[i].x) * k2)) + v[i].y;
+          m_l = v[i].x;
+        } else {
+          z_l += v[i].y * exp2f_approx((v[i].x - m_l) * k2);
+        }
+      }
     }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) first = min(first, __shfl_xor_sync(0xffffffffu, first, off));
-    if (first == INT_MAX) return 0;
-    float x[8];
-    seg_load<T>(row, p.V, false, first, x);
-    int hit = 8;
-#pragma unroll
-    for (int i = 7; i >= 0; --i)
-      if (isnan(M) ? isnan(x[i]) : x[i] == INFINITY) hit = i;
-    const unsigned bal = __ballot_sync(0xffffffffu, hit < 8);
-    const int l0 = __ffs(bal) - 1;
-    return first * SEG + 8 * l0 + __shfl_sync(0xffffffffu, hit, l0);
   }
-  // weights of this lane's segments in the row's scale, their block sum, and
-  // an inclusive scan over the lanes (segment order)
-  float wsum = 0.f;
-  for (int g = gb; g < ge; ++g) {
-    const float2 ms = __ldcg(seg_row + g);
-    if (ms.x != -INFINITY) wsum += ms.y * exp2f_approx((ms.x - M) * p.k2);
-  }
-  float inc = wsum;
 #pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const float y = __shfl_up_sync(0xffffffffu, inc, off);
-    if (lane >= off) inc += y;
+  for (int off = 16; off > 0; off >>= 1) {
+    first_nan = min(first_nan, __shfl_xor_sync(0xffffffffu, first_nan, off));
+    first_inf = min(first_inf, __shfl_xor_sync(0xffffffffu, first_inf, off));
   }
-  const float Z = __shfl_sync(0xffffffffu, inc, 31);
+  if (first_nan != INT_MAX || first_inf != INT_MAX) {
+    // degenerate: the first NaN, else the first +inf (the argmax order)
+    const bool want_nan = first_nan != INT_MAX;
+    const int g = want_nan ? first_nan : first_inf;
+    for (int k = 0; k < 4; ++k) {
+      float x[8];
+      sub_load<T>(row, p.V, false, 4 * int64_t(g) + k, x);
+      int hit = 8;
+#pragma unroll
+      for (int i = 7; i >= 0; --i)
+        if (want_nan ? isnan(x[i]) : x[i] == INFINITY) hit = i;
+      const unsigned bal = __ballot_sync(0xffffffffu, hit < 8);
+      if (bal) {
+        const int l0 = __ffs(bal) - 1;
+        return g * SEG + k * SUB + 8 * l0 + __shfl_sync(0xffffffffu, hit, l0);
+      }
+    }
+    return g * SEG;
+  }
+  float M = m_l;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  if (M == -INFINITY) return 0;  // every value -inf: the argmax is index 0
+  float Z = m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - M) * k2);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Z += __shfl_xor_sync(0xffffffffu, Z, off);
   const float uc = u > 0.f ? fminf(u, 1.f) : 0.f;  // NaN and negatives count as 0
   const float t = uc * Z;
-  const unsigned cross = __ballot_sync(0xffffffffu, inc > t);
-  int gs = -1;         // segment holding the draw
-  float r = 0.f;       // what is left of t at the start of that segment, in its own scale
-  bool tail = false;   // no crossing: take the last value of positive weight
-  if (cross) {
-    const int L = __ffs(cross) - 1;
-    if (lane == L) {
-      float acc = inc - wsum;
-      int last = -1;
-      float last_r = 0.f;
-      for (int g = gb; g < ge; ++g) {
-        const float2 ms = __ldcg(seg_row + g);
-        if (ms.x == -INFINITY) continue;
-        const float sc = exp2f_approx((ms.x - M) * p.k2);
-        const float c = ms.y * sc;
-        if (c > 0.f) {
-          last = g;
-          last_r = fmaxf(t - acc, 0.f) / sc;
-        }
-        if (acc + c > t) {
-          gs = g;
-          r = fmaxf(t - acc, 0.f) / sc;  // >= 0: the draw has positive weight
-          break;
-        }
-        acc += c;
-      }
-      if (gs < 0) {
-        gs = last;
-        r = last_r;
-        tail = true;
-      }
+  // ---- pass 2: running sums in segment order up to the crossing
+  int gs = -1;        // segment holding the draw
+  float r = 0.f;      // what is left of t at the start of that segment, in its own scale
+  bool tail = true;   // no crossing found: take the last value of positive weight
+  int last = -1;      // last segment of positive weight seen
+  float carry = 0.f;
+  for (int base = 0; base < nseg && gs < 0; base += 256) {
+    float2 v[8];
+    seg_batch(seg_row, nseg, base, v);
+    float c[8], ls = 0.f;
+    int llast = -1;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      c[i] = v[i].x != -INFINITY ? v[i].y * exp2f_approx((v[i].x - M) * k2) : 0.f;
+      ls += c[i];
+      if (c[i] > 0.f) llast = base + 8 * lane + i;
     }
-    gs = __shfl_sync(0xffffffffu, gs, L);
-    r = __shfl_sync(0xffffffffu, r, L);
-    tail = __shfl_sync(0xffffffffu, tail, L);
-  } else {
-    // t >= Z (u = 1, or rounding): the last segment of positive weight
-    int last = -1;
-    for (int g = gb; g < ge; ++g) {
-      const float2 ms = __ldcg(seg_row + g);
-      if (ms.x != -INFINITY && ms.y * exp2f_approx((ms.x - M) * p.k2) > 0.f) last = g;
+    float inc = ls;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, inc, off);
+      if (lane >= off) inc += y;
     }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, off));
-    gs = last;
-    tail = true;
+    for (int off = 16; off > 0; off >>= 1) llast = max(llast, __shfl_xor_sync(0xffffffffu, llast, off));
+    const int last_before = last;
+    if (llast >= 0) last = llast;
+    const unsigned cross = __ballot_sync(0xffffffffu, carry + inc > t);
+    if (cross) {
+      const int L = __ffs(cross) - 1;
+      int g_hit = -1, g_prev = -1;
+      float r_hit = 0.f;
+      if (lane == L) {
+        float acc = carry + inc - ls;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (g_hit < 0 && c[i] > 0.f) {
+            if (acc + c[i] > t) {
+              g_hit = base + 8 * lane + i;
+              r_hit = fmaxf(t - acc, 0.f) / exp2f_approx((v[i].x - M) * k2);  // >= 0: positive weight
+            } else {
+              g_prev = base + 8 * lane + i;
+            }
+          }
+          acc += c[i];
+        }
+      }
+      g_hit = __shfl_sync(0xffffffffu, g_hit, L);
+      r_hit = __shfl_sync(0xffffffffu, r_hit, L);
+      g_prev = __shfl_sync(0xffffffffu, g_prev, L);
+      if (g_hit >= 0) {
+        gs = g_hit;
+        r = r_hit;
+        tail = false;
+      } else {
+        // rounding left the crossing just past lane L's segments: the last
+        // positive one up to there
+        int lp = -1;
+        for (int i = 0; i < 8; ++i)
+          if (c[i] > 0.f && base + 8 * lane + i < base + 8 * L) lp = base + 8 * lane + i;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, off));
+        gs = g_prev >= 0 ? g_prev : (lp >= 0 ? lp : last_before);
+      }
+    }
+    carry += __shfl_sync(0xffffffffu, inc, 31);
   }
+  if (gs < 0) gs = last;  // t >= every running sum (u = 1, or rounding)
   if (gs < 0) return 0;
-  // the segment again, in index order, in its own scale
+  // ---- the crossing segment again, step by step in index order, in its own scale
   const float m = __ldcg(seg_row + gs).x;
-  float x[8];
-  seg_load<T>(row, p.V, p.vec_ok, gs, x);
-  float w[8], ls = 0.f;
+  float acc = 0.f;
+  int last_i = -1;  // last value of positive weight seen (index)
+  for (int k = 0; k < 4; ++k) {
+    float x[8];
+    sub_load<T>(row, p.V, p.vec_ok, 4 * int64_t(gs) + k, x);
+    float w[8], ls = 0.f;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    w[i] = exp2f_approx((x[i] - m) * p.k2);
-    ls += w[i];
-  }
-  float linc = ls;
+    for (int i = 0; i < 8; ++i) {
+      w[i] = exp2f_approx((x[i] - m) * k2);
+      ls += w[i];
+    }
+    float linc = ls;
 #pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const float y = __shfl_up_sync(0xffffffffu, linc, off);
-    if (lane >= off) linc += y;
-  }
-  int pick = -1;
-  const unsigned lc = tail ? 0u : __ballot_sync(0xffffffffu, linc > r);
-  if (lc) {
-    const int L = __ffs(lc) - 1;
-    if (lane == L) {
-      float acc = linc - ls;
-      for (int i = 0; i < 8; ++i) {
-        acc += w[i];
-        if (w[i] > 0.f) pick = i;
-        if (acc > r) {
-          pick = i;
-          break;
+    for (int off = 1; off < 32; off <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, linc, off);
+      if (lane >= off) linc += y;
+    }
+    const int base_e = gs * SEG + k * SUB + 8 * lane;
+    const unsigned lc = tail ? 0u : __ballot_sync(0xffffffffu, acc + linc > r);
+    if (lc) {
+      const int L = __ffs(lc) - 1;
+      int pick = -1;
+      if (lane == L) {
+        float a = acc + linc - ls;
+        bool done = false;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          a += w[i];
+          if (!done && w[i] > 0.f) {
+            pick = base_e + i;
+            done = a > r;
+          }
         }
       }
+      pick = __shfl_sync(0xffffffffu, pick, L);
+      if (pick >= 0) return pick;
     }
-    pick = __shfl_sync(0xffffffffu, pick, L);
-    return gs * SEG + 8 * (__ffs(lc) - 1) + pick;
-  }
-  // the segment's last value of positive weight
-  int li = -1;
+    int li = -1;
 #pragma unroll
-  for (int i = 0; i < 8; ++i)
-    if (w[i] > 0.f) li = i;
-  const unsigned has = __ballot_sync(0xffffffffu, li >= 0);
-  if (!has) return gs * SEG;
-  const int L = 31 - __clz(has);
-  return gs * SEG + 8 * L + __shfl_sync(0xffffffffu, li, L);
+    for (int i = 0; i < 8; ++i)
+      if (w[i] > 0.f) li = base_e + i;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) li = max(li, __shfl_xor_sync(0xffffffffu, li, off));
+    if (li >= 0) last_i = li;
+    acc += __shfl_sync(0xffffffffu, linc, 31);
+  }
+  // no crossing in the segment (t at its very end, or u = 1): its last value
+  // of positive weight
+  return last_i >= 0 ? last_i : gs * SEG;
 }
 
 template <typename T>
-__global__ void __launch_bounds__(SAMPLE_THREADS) vocab_sample_stats_kernel(const SampleParams p) {
-  const int64_t row = blockIdx.x / p.ncta_row;
+__global__ void __launch_bounds__(SAMPLE_THREADS, sizeof(T) == 2 ? 6 : 4) vocab_sample_stats_kernel(const SampleParams p) {
+  const int64_t r = blockIdx.x / p.ncta_row;
   const int c = blockIdx.x % p.ncta_row;
-  const T *base = static_cast<const T *>(p.logits) + row * p.row_stride;
   const int64_t g0 = int64_t(c) * p.seg_per_cta, g1 = std::min<int64_t>(p.nseg, g0 + p.seg_per_cta);
-  sample_stats<T>(p, base, p.seg + row * p.nseg, g0, g1);
+  sample_stats<T>(p, static_cast<const T *>(p.logits) + r * p.row_stride, p.seg + r * p.nseg, g0, g1);
+  // the selection grid may launch as this one drains
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// Stage 2, one warp per row, chained to stage 1 by programmatic dependent
+// launch (it waits until stage 1 has completed).
 template <typename T>
 __global__ void __launch_bounds__(256) vocab_sample_select_kernel(const SampleParams p, int64_t rows, int32_t *out) {
-  const int64_t row = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
-  if (row >= rows) return;
-  const T *base = static_cast<const T *>(p.logits) + row * p.row_stride;
-  const int idx = sample_select_warp<T>(p, base, p.seg + row * p.nseg, __ldg(p.u + row));
-  if ((threadIdx.x & 31) == 0) out[row] = idx;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int64_t r = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  const int idx = sample_select_warp<T>(p, static_cast<const T *>(p.logits) + r * p.row_stride, p.seg + r * p.nseg,
+                                        __ldg(p.u + r));
+  if ((threadIdx.x & 31) == 0) out[r] = idx;
 }
 
 // ------------------------------------------------------------------ tree walk
@@ -772,8 +882,7 @@ __global__ void __launch_bounds__(TAIL_THREADS) kv_compact_kernel(const KVParams
 
 struct StepParams {
   ArgmaxParams am;
-  SampleParams sp;
-  bool sampled;  // predictions are draws at temperature tau (sp), not argmaxes (am)
+  SampleParams sp;  // the draws at temperature tau (sampled step)
   TreeParams tr;
   KVParams kv;
   int32_t max_path;
@@ -805,28 +914,44 @@ __global__ void __launch_bounds__(ARGMAX_THREADS) verify_rows_kernel(const StepP
     p.pred[rb + i] = row_idx;
 }
 
-// Launch 1 of the sampled verification tail. grid.x = B * T_max * ncta_row:
-// (sequence, tree node, segment range); padding nodes return at once. Stage 1
-// of the draw (segment statistics) of the node's row.
+// Launches 1 and 2 of the sampled verification tail: stage 1 over the rows of
+// tree nodes (grid.x = B * T_max * ncta_row; padding nodes return at once),
+// then stage 2 (one warp per node row; grid.x = B * T_max / 8 rounded up),
+// which writes the draws as the predictions.
 template <typename T>
-__global__ void __launch_bounds__(SAMPLE_THREADS) verify_sample_rows_kernel(const StepParams p) {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+__global__ void __launch_bounds__(SAMPLE_THREADS, sizeof(T) == 2 ? 6 : 4) verify_sample_stats_kernel(const StepParams p) {
   const int ncta = p.sp.ncta_row;
-  const int c = blockIdx.x % ncta;
   const int rowg = blockIdx.x / ncta;
   const int b = rowg / p.tr.T_max, i = rowg % p.tr.T_max;
   const int tl = __ldg(p.tr.tree_len + b);
+  if (tl >= 1 && tl <= p.tr.T_max && i < tl) {
+    const int64_t r = int64_t(b) * p.tr.T_max + i;
+    const int64_t g0 = int64_t(blockIdx.x % ncta) * p.sp.seg_per_cta;
+    const int64_t g1 = std::min<int64_t>(p.sp.nseg, g0 + p.sp.seg_per_cta);
+    sample_stats<T>(p.sp, static_cast<const T *>(p.sp.logits) + r * p.sp.row_stride, p.sp.seg + r * p.sp.nseg,
+                    g0, g1);
+  }
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) verify_sample_select_kernel(const StepParams p) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int rowg = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int b = rowg / p.tr.T_max, i = rowg % p.tr.T_max;
+  if (b >= p.tr.B) return;
+  const int tl = __ldg(p.tr.tree_len + b);
   if (tl < 1 || tl > p.tr.T_max || i >= tl) return;
   const int64_t r = int64_t(b) * p.tr.T_max + i;
-  const T *row = static_cast<const T *>(p.sp.logits) + r * p.sp.row_stride;
-  const int64_t g0 = int64_t(c) * p.sp.seg_per_cta, g1 = std::min<int64_t>(p.sp.nseg, g0 + p.sp.seg_per_cta);
-  sample_stats<T>(p.sp, row, p.sp.seg + r * p.sp.nseg, g0, g1);
+  const int idx = sample_select_warp<T>(p.sp, static_cast<const T *>(p.sp.logits) + r * p.sp.row_stride,
+                                        p.sp.seg + r * p.sp.nseg, __ldg(p.sp.u + r));
+  if ((threadIdx.x & 31) == 0) p.pred[r] = idx;
 }
 
 // Launch 2 of the verification tail, one CTA per sequence, chained to launch 1
 // by programmatic dependent launch (it may start early and waits until launch
 // 1 has completed): the acceptance walk, its outputs, and the KV compaction.
-template <typename LT>
 __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepParams p) {
   __shared__ int32_t s_path[65];
   __shared__ int64_t s_src[65], s_dst[65];
@@ -836,16 +961,6 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
   const int64_t rb = int64_t(b) * Tm;
   const int T = __ldg(p.tr.tree_len + b);
   const int L = __ldg(p.tr.kv_len + b);
-  if (p.sampled && T >= 1 && T <= Tm) {
-    // stage 2 of the draws: one warp per node row
-    for (int i = threadIdx.x >> 5; i < T; i += TAIL_THREADS / 32) {
-      const int64_t r = rb + i;
-      const LT *row = static_cast<const LT *>(p.sp.logits) + r * p.sp.row_stride;
-      const int idx = sample_select_warp<LT>(p.sp, row, p.sp.seg + r * p.sp.nseg, __ldg(p.sp.u + r));
-      if ((threadIdx.x & 31) == 0) p.pred[r] = idx;
-    }
-    __syncthreads();
-  }
   if (threadIdx.x < 32) {
     WalkOut w{-1, 0};
     if (T < 1 || T > Tm) w.bad = DREAMS_DATA_BAD_TREE_LEN;
@@ -906,6 +1021,26 @@ SamplePlan plan_sample(int64_t rows, int64_t V) {
 }
 
 size_t sample_ws(int64_t rows, int64_t V) { return align_up(size_t(rows) * size_t((V + SEG - 1) / SEG) * 8, 256); }
+
+// Launches `kernel` as a programmatic dependent of the previous launch on the stream.
+template <typename... Args>
+dreams_status_t launch_dependent(void (*kernel)(Args...), dim3 grid, dim3 block, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args...);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
+  return check_launch();
+}
 
 // Checks and fills the sampling parameters shared by both entry points.
 bool sample_params(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V, int64_t row_stride,
@@ -1084,8 +1219,7 @@ extern "C" dreams_status_t dreams_verify_step(const void *logits, dreams_dtype_t
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const cudaError_t e = dtype == DREAMS_F32 ? cudaLaunchKernelEx(&cfg, verify_tail_kernel<float>, p)
-                                             : cudaLaunchKernelEx(&cfg, verify_tail_kernel<__nv_bfloat16>, p);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, verify_tail_kernel, p);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return DREAMS_ERR_CUDA;
@@ -1116,15 +1250,13 @@ extern "C" dreams_status_t dreams_vocab_sample(const void *logits, dreams_dtype_
     return DREAMS_ERR_INVALID_ARG;
   if (ctas > INT_MAX || (rows + 7) / 8 > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 g1(static_cast<unsigned>(ctas)), g2(static_cast<unsigned>((rows + 7) / 8));
-  if (dtype == DREAMS_F32) {
-    vocab_sample_stats_kernel<float><<<g1, SAMPLE_THREADS, 0, s>>>(p);
-    vocab_sample_select_kernel<float><<<g2, 256, 0, s>>>(p, rows, out_idx);
-  } else {
-    vocab_sample_stats_kernel<__nv_bfloat16><<<g1, SAMPLE_THREADS, 0, s>>>(p);
-    vocab_sample_select_kernel<__nv_bfloat16><<<g2, 256, 0, s>>>(p, rows, out_idx);
-  }
-  return check_launch();
+  const dim3 grid(static_cast<unsigned>(ctas)), g2(static_cast<unsigned>((rows + 7) / 8));
+  if (dtype == DREAMS_F32) vocab_sample_stats_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  else vocab_sample_stats_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  dreams_status_t st = check_launch();
+  if (st != DREAMS_OK) return st;
+  if (dtype == DREAMS_F32) return launch_dependent(vocab_sample_select_kernel<float>, g2, dim3(256), s, p, rows, out_idx);
+  return launch_dependent(vocab_sample_select_kernel<__nv_bfloat16>, g2, dim3(256), s, p, rows, out_idx);
 }
 
 extern "C" size_t dreams_verify_step_sampled_workspace_size(const dreams_tree_t *tree, int64_t V) {
@@ -1155,7 +1287,6 @@ extern "C" dreams_status_t dreams_verify_step_sampled(
   if (!sample_params(logits, dtype, rows, V, row_stride, temperature, uniforms, ws, p.sp, ctas))
     return DREAMS_ERR_INVALID_ARG;
   if (ctas > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
-  p.sampled = true;
   int32_t *ws_pred = reinterpret_cast<int32_t *>(ws + sample_ws(rows, V));
   p.pred = sample_out != nullptr ? sample_out : ws_pred;
   p.pred_in_ws = false;
@@ -1166,27 +1297,15 @@ extern "C" dreams_status_t dreams_verify_step_sampled(
   p.new_kv_len = new_kv_len;
   p.status = status_word;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid(static_cast<unsigned>(ctas));
-  if (dtype == DREAMS_F32) verify_sample_rows_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
-  else verify_sample_rows_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  const dim3 grid(static_cast<unsigned>(ctas)), g2(static_cast<unsigned>((rows + 7) / 8));
+  if (dtype == DREAMS_F32) verify_sample_stats_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  else verify_sample_stats_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
   dreams_status_t st = check_launch();
   if (st != DREAMS_OK) return st;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(unsigned(tree->B));
-  cfg.blockDim = dim3(TAIL_THREADS);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  const cudaError_t e = dtype == DREAMS_F32 ? cudaLaunchKernelEx(&cfg, verify_tail_kernel<float>, p)
-                                             : cudaLaunchKernelEx(&cfg, verify_tail_kernel<__nv_bfloat16>, p);
-  if (e != cudaSuccess) {
-    set_last_cuda_error(e);
-    return DREAMS_ERR_CUDA;
-  }
-  return check_launch();
+  st = dtype == DREAMS_F32 ? launch_dependent(verify_sample_select_kernel<float>, g2, dim3(256), s, p)
+                           : launch_dependent(verify_sample_select_kernel<__nv_bfloat16>, g2, dim3(256), s, p);
+  if (st != DREAMS_OK) return st;
+  return launch_dependent(verify_tail_kernel, dim3(unsigned(tree->B)), dim3(TAIL_THREADS), s, p);
 }
 
 // ------------------------------------------------------------------ no-allocation argmax

@@ -197,3 +197,34 @@ def test_verify_step_sampled_low_temperature_is_greedy(dreams):
     for key in ("accept_len", "path", "out_tokens", "new_kv_len"):
         assert torch.equal(r_s[key], r_g[key]), key
     assert torch.equal(g1["k"], g2["k"]) and torch.equal(g1["v"], g2["v"])
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_sample_split_rows_repeat(dreams, dtype):
+    """Few long rows, each split between CTAs; two calls on one workspace agree."""
+    rng = np.random.default_rng(23)
+    rows, V = 5, 300_001
+    x = (2.0 * rng.standard_normal((rows, V))).astype(np.float32)
+    u = rng.uniform(0, 1, rows).astype(np.float32)
+    t = torch.from_numpy(x) if dtype == "f32" else W.bf16(x)
+    need = dreams._lib().dreams_vocab_sample_workspace_size(rows, V)
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    ut = torch.from_numpy(u).cuda()
+    a = dreams.vocab_sample(t.cuda(), 1.0, ut, workspace=ws).cpu().numpy()
+    ws.fill_(0xA5)  # the workspace holds no state: garbage in it changes nothing
+    b = dreams.vocab_sample(t.cuda(), 1.0, ut, workspace=ws).cpu().numpy()
+    np.testing.assert_array_equal(a, b)
+    ref = oracle.sample(W.bits(t) if dtype == "bf16" else x, 1.0, u, bf16_bits=dtype == "bf16")
+    _check_draws(t.float().numpy(), 1.0, u, a, ref)
+
+
+def test_sample_workspace_reused_across_shapes(dreams):
+    """One workspace for calls of different shapes (the binding caches one per stream)."""
+    rng = np.random.default_rng(24)
+    need = max(dreams._lib().dreams_vocab_sample_workspace_size(r, V) for r, V in ((3, 200_000), (40, 32000)))
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    for rows, V in ((3, 200_000), (40, 32000), (3, 200_000), (7, 1000)):
+        x = rng.standard_normal((rows, V)).astype(np.float32)
+        u = rng.uniform(0, 1, rows).astype(np.float32)
+        got = dreams.vocab_sample(torch.from_numpy(x).cuda(), 1.0, torch.from_numpy(u).cuda(), workspace=ws)
+        _check_draws(x, 1.0, u, got.cpu().numpy(), oracle.sample(x, 1.0, u))
