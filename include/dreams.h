@@ -261,6 +261,32 @@ dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dt
                                            dreams_stream_t stream);
 
 /*
+ * The LM head with its argmax fused: the target's greedy prediction per node
+ * straight from its final hidden states (Sec. 2 "Speculative decoding" at
+ * temperature 0), without writing the logits:
+ *     logits[r][v] = sum_k hidden[r][k] * weight[v][k]     (f32 accumulation)
+ *     out_idx[r]   = argmax_v logits[r][v]  (the order of dreams_vocab_argmax)
+ *     out_max[r]   = logits[r][out_idx[r]]  (may be NULL)
+ * hidden: bf16 [rows, hidden_dim] with row stride ld_hidden; weight: bf16
+ * [V, hidden_dim] with row stride ld_weight (the usual [vocab, hidden] layout).
+ * hidden_dim must be a multiple of 64, both strides multiples of 8 elements,
+ * both pointers 16-byte aligned. The products of bf16 values are exact in
+ * f32; the f32 sums run in the tensor cores' order, so a row whose two largest
+ * logits lie within rounding of each other may get either index. Two launches:
+ * a persistent tcgen05 GEMM (128 x 256 tiles, the argmax of each tile merged
+ * into a 64-bit slot per row with atomicMax), then a small kernel that writes
+ * the indices and resets the slots. The workspace holds the slots: zero-fill
+ * it once when it is allocated; every call leaves it zero-filled. A wait that
+ * times out inside the GEMM flags DREAMS_DATA_TIMEOUT in status_word (may be
+ * NULL).
+ */
+size_t dreams_lm_head_argmax_workspace_size(int64_t rows);
+dreams_status_t dreams_lm_head_argmax(const void *hidden, int64_t rows, int64_t hidden_dim, int64_t ld_hidden,
+                                      const void *weight, int64_t V, int64_t ld_weight, int32_t *out_idx,
+                                      float *out_max, void *workspace, size_t workspace_bytes,
+                                      int32_t *status_word, dreams_stream_t stream);
+
+/*
  * Row-wise argmax for callers that cannot allocate device memory. The paper
  * has no counterpart to this call; it exists for integration. Some callers
  * cannot allocate, or cannot hand out a workspace, when the argmax runs: a

@@ -20,6 +20,9 @@ paper passage its C routine follows:
   by inverse transform of softmax(x / tau) with a caller-supplied uniform
   (Sec. 2 "Speculative decoding": drafts are checked against the target's own
   sampling; Table 2, Temperature = 1).
+* :func:`lm_head_argmax` -- the target's greedy prediction from its final
+  hidden states: argmax over the vocabulary of H W^T, in fp64 (numpy's matmul
+  as the product step), the same total order as :func:`argmax`.
 * :func:`accept_path` -- sequential acceptance with the target's token
   replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
 * :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
@@ -190,6 +193,22 @@ def sample(logits, temperature: float, u, V: Optional[int] = None, bf16_bits: bo
         x = _c(x, np.float32)
         _load().oracle_sample_f32(_ptr(x), rows, V, x.shape[1], float(temperature), _ptr(uu), _ptr(out))
     return out
+
+
+def lm_head_argmax(hidden_bits, weight_bits):
+    """(indices, maxima, logits) of the LM head: logits = H W^T in float64 from
+    bf16 bit patterns (uint16 [rows, K] and [V, K]); argmax with the lowest
+    index among equal values (numpy's argmax; NaN first, as torch)."""
+    h = _bf16_to_f64(hidden_bits)
+    w = _bf16_to_f64(weight_bits)
+    logits = np.matmul(h, w.T)
+    idx = np.argmax(logits, axis=1).astype(np.int32)
+    return idx, logits[np.arange(logits.shape[0]), idx], logits
+
+
+def _bf16_to_f64(bits):
+    b = np.ascontiguousarray(bits, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
 def accept_path(am, parent, tokens, tree_len, kv_len, max_path: int):

@@ -86,6 +86,8 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, p, p, p, p,
                                                           p, p, sz, p, p]),
                     "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
+                    "dreams_lm_head_argmax_workspace_size": (sz, [i64]),
+                    "dreams_lm_head_argmax": (ctypes.c_int, [p, i64, i64, i64, p, i64, i64, p, p, p, sz, p, p]),
                     "dreams_vocab_sample_workspace_size": (sz, [i64, i64]),
                     "dreams_vocab_sample": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, f32, p, p, p, sz, p]),
                     "dreams_verify_step_sampled_workspace_size": (sz, [ptr, i64]),
@@ -328,6 +330,38 @@ def vocab_sample(logits: torch.Tensor, temperature: float, uniforms: torch.Tenso
         _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
     _check("dreams_vocab_sample", st)
     return out
+
+
+def lm_head_argmax(hidden: torch.Tensor, weight: torch.Tensor, out: Optional[torch.Tensor] = None,
+                   out_max: Optional[torch.Tensor] = None, want_max: bool = False,
+                   workspace: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+                   stream=None):
+    """argmax over the vocabulary of hidden @ weight.T (bf16 [rows, K] and
+    [V, K], f32 accumulation) without writing the logits. Returns the indices
+    (int32 [rows]) and, with ``want_max``, the maximum logits (f32 [rows])."""
+    for n, t in (("hidden", hidden), ("weight", weight)):
+        if t.dtype != torch.bfloat16 or t.dim() != 2 or t.stride(1) != 1:
+            raise TypeError(f"{n} must be a 2-D bf16 tensor with contiguous rows")
+    if weight.device != hidden.device or weight.shape[1] != hidden.shape[1]:
+        raise ValueError("hidden and weight must share the device and the hidden size")
+    rows, K = int(hidden.shape[0]), int(hidden.shape[1])
+    V = int(weight.shape[0])
+    dev = hidden.device
+    if out is None:
+        out = torch.empty(rows, dtype=torch.int32, device=dev)
+    _need(out, "out", torch.int32, dev)
+    if out_max is None and want_max:
+        out_max = torch.empty(rows, dtype=torch.float32, device=dev)
+    if out_max is not None:
+        _need(out_max, "out_max", torch.float32, dev)
+    need = int(_lib().dreams_lm_head_argmax_workspace_size(rows))
+    if workspace is None:
+        workspace = _workspace("lm_head", need, dev, stream)
+    st = _lib().dreams_lm_head_argmax(_ptr(hidden), rows, K, int(hidden.stride(0)), _ptr(weight), V,
+                                      int(weight.stride(0)), _ptr(out), _ptr(out_max), _ptr(workspace),
+                                      0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
+    _check("dreams_lm_head_argmax", st)
+    return (out, out_max) if want_max or out_max is not None else out
 
 
 def _walk_outputs(B: int, max_path: int, dev):

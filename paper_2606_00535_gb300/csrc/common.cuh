@@ -1,5 +1,6 @@
 // common.cuh -- device helpers shared by the library's kernels (sm_103a).
 #pragma once
+#include <limits.h>
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -40,37 +41,21 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
 }
 
 // 16-byte global -> shared copy; src_bytes == 0 zero-fills the destination.
-__device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
-}
-
-__device__ __forceinline__ void ldmatrix_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                            uint32_t &r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                                  uint32_t &r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
+// Order-preserving integer key of an f32 bit pattern for the argmax order:
+// greater value -> greater key, +0 == -0, NaN above every number.
+__device__ __forceinline__ int order_key(uint32_t u) {
+  const uint32_t mag = u & 0x7fffffffu;
+  if (mag > 0x7f800000u) return INT_MAX;  // NaN
+  if (mag == 0u) return 0;                // +0 and -0
+  const int s = static_cast<int>(u);
+  return s ^ ((s >> 31) & 0x7fffffff);
 }
 
-// D(16x8 f32) += A(16x16 bf16, row) * B(16x8 bf16, col)
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                               uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+// (key, index) packed so that a 64-bit max keeps the greater key, then the
+// lower index.
+__device__ __forceinline__ unsigned long long pack_key_idx(int key, int idx) {
+  return (static_cast<unsigned long long>(static_cast<uint32_t>(key) ^ 0x80000000u) << 32) |
+         static_cast<unsigned long long>(~static_cast<uint32_t>(idx));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {

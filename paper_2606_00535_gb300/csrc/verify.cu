@@ -41,14 +41,6 @@ namespace {
 constexpr int ARGMAX_THREADS = 256;
 constexpr int TAIL_THREADS = 256;
 
-// ------------------------------------------------------------------ keys
-__device__ __forceinline__ int order_key(uint32_t u) {
-  const uint32_t mag = u & 0x7fffffffu;
-  if (mag > 0x7f800000u) return INT_MAX;  // NaN
-  if (mag == 0u) return 0;                // +0 and -0
-  const int s = static_cast<int>(u);
-  return s ^ ((s >> 31) & 0x7fffffff);
-}
 
 __device__ __forceinline__ bool better(int ka, int ia, int kb, int ib) {
   return ka > kb || (ka == kb && ia < ib);
@@ -193,10 +185,6 @@ __device__ void block_argmax(const T *row, int64_t begin, int64_t end, bool vec_
   __syncthreads();
 }
 
-__device__ __forceinline__ unsigned long long pack_key_idx(int key, int idx) {
-  return (static_cast<unsigned long long>(static_cast<uint32_t>(key) ^ 0x80000000u) << 32) |
-         static_cast<unsigned long long>(~static_cast<uint32_t>(idx));
-}
 
 // Combines one chunk's winner into the row's slot. Returns true (and the
 // row's index) in the CTA that finished the row last.
