@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sampled", action="store_true",
                     help="skip the extra timing of the temperature-1 verification tail")
+    ap.add_argument("--no-lm-head", action="store_true",
+                    help="skip the extra timing of the LM head with the fused argmax")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
     ap.add_argument("--load-seconds", type=float, default=1.0,
                     help="untimed steps run while the clock sampler starts (0 under a profiler)")
@@ -91,6 +93,16 @@ def measured_traffic(kernel: str, workload: str):
     if sha != rec["source_sha256"] or rec["workload"] != workload:
         return None
     return int(rec["dram_bytes_per_launch"])
+
+
+def bf16_peaks():
+    """(burst, sustained) dense bf16 TFLOP/s from MEASURED_PEAKS.json, else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"])
+    except (OSError, KeyError, ValueError):
+        return 1900.0, 1700.0
 
 
 def peaks():
@@ -344,6 +356,40 @@ def run_dreams(args, rank, world, local):
         sampled = {"us": round(sampled_us, 2), "temperature": 1.0, "launches": dreams.VERIFY_STEP_SAMPLED_LAUNCHES,
                    "launch": "eager", "GBps": round(argmax_bytes(w) / (sampled_us * 1e-6) / 1e9, 1)}
 
+    # ---- the LM head with its argmax fused (the logits never reach HBM), on
+    # the tree rows of this workload: hidden size Hq * D, random bf16 weights
+    lm_head = None
+    if not args.no_lm_head:
+        rows = int(w.tree_len.sum())
+        hid = w.Hq * w.D
+        gen = torch.Generator(device=dev).manual_seed(11)
+        Hs = torch.randn((rows, hid), device=dev, generator=gen).to(torch.bfloat16)
+        Wt = (torch.randn((w.V, hid), device=dev, generator=gen) * hid ** -0.5).to(torch.bfloat16)
+        lm_out = torch.empty(rows, dtype=torch.int32, device=dev)
+        ws_lm = torch.zeros(dreams._lib().dreams_lm_head_argmax_workspace_size(rows), dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            dreams.lm_head_argmax(Hs, Wt, out=lm_out, workspace=ws_lm, status=status)
+        Kl = max(3, min(K, 20))
+        l0 = torch.cuda.Event(enable_timing=True)
+        l1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        l0.record(stream)
+        for _ in range(Kl):
+            dreams.lm_head_argmax(Hs, Wt, out=lm_out, workspace=ws_lm, status=status)
+        l1.record(stream)
+        barrier()
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item()):#x} (lm head)")
+        lm_us = l0.elapsed_time(l1) / Kl * 1000.0
+        tflops = 2.0 * rows * hid * w.V / (lm_us * 1e-6) / 1e12
+        bf16_burst, bf16_sust = bf16_peaks()
+        lm_head = {"us": round(lm_us, 1), "rows": rows, "hidden": hid, "V": w.V, "bound": "tensor",
+                   "tflops": round(tflops, 1), "peak_tflops_sustained": bf16_sust, "peak_tflops_burst": bf16_burst,
+                   "frac_of_sustained": round(tflops / bf16_sust, 4), "frac_of_burst": round(tflops / bf16_burst, 4),
+                   "weight_GBps": round(w.V * hid * 2 / (lm_us * 1e-6) / 1e9, 1), "launches": 2,
+                   "note": "timed back to back over ~10 ms: the sustained peak applies"}
+        del Hs, Wt
+
     ab, gb = attn_bytes(w), argmax_bytes(w)
     attn_avg_ms = sum(attn_ms) / K
     tail_avg_ms = sum(tail_ms) / K
@@ -368,6 +414,8 @@ def run_dreams(args, rank, world, local):
     if sampled is not None:
         sampled["frac_measured_hbm"] = round(sampled["GBps"] / peak, 4)
         kernels["verify_step_sampled"] = sampled
+    if lm_head is not None:
+        kernels["lm_head_argmax"] = lm_head
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
