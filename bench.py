@@ -52,6 +52,8 @@ def parse():
                     help="skip the extra timing of the temperature-1 verification tail")
     ap.add_argument("--no-lm-head", action="store_true",
                     help="skip the extra timing of the LM head with the fused argmax")
+    ap.add_argument("--no-importance", action="store_true",
+                    help="skip the extra timing of the visual-token importance (Eq. 2) on a LLaVA-7B-shaped prefill")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
     ap.add_argument("--load-seconds", type=float, default=1.0,
                     help="untimed steps run while the clock sampler starts (0 under a profiler)")
@@ -390,6 +392,39 @@ def run_dreams(args, rank, world, local):
                    "note": "timed back to back over ~10 ms: the sustained peak applies"}
         del Hs, Wt
 
+    # ---- visual-token importance (Eq. 2) + top-r on the final-layer attention
+    # of a LLaVA-7B-shaped prefill: 32 heads, 3392 positions, 2880 visual
+    # tokens after a 35-token prompt, keep r = 576; synthetic causal softmax
+    # weights, two rotating copies (736 MB each, larger than L2)
+    importance = None
+    if not args.no_importance:
+        Hh, Qn, v0, nv, rk = 32, 3392, 35, 2880, 576
+        gen = torch.Generator(device=dev).manual_seed(13)
+        imp_in = []
+        for _ in range(2):
+            sc = torch.randn((1, Hh, Qn, Qn), device=dev, generator=gen)
+            causal = torch.ones((Qn, Qn), dtype=torch.bool, device=dev).tril()
+            imp_in.append(torch.softmax(sc.masked_fill_(~causal, float("-inf")), dim=-1).to(torch.bfloat16))
+            del sc, causal
+        ws_imp = torch.zeros(dreams._lib().dreams_visual_importance_workspace_size(1, Hh, Qn, nv), dtype=torch.uint8,
+                             device=dev)
+        for i in range(3):
+            dreams.visual_importance(imp_in[i % 2], v0, nv, rk, workspace=ws_imp)
+        Ki = max(3, min(K, 20))
+        i0 = torch.cuda.Event(enable_timing=True)
+        i1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        i0.record(stream)
+        for i in range(Ki):
+            dreams.visual_importance(imp_in[i % 2], v0, nv, rk, workspace=ws_imp)
+        i1.record(stream)
+        barrier()
+        imp_us = i0.elapsed_time(i1) / Ki * 1000.0
+        imp_bytes = Hh * Qn * nv * 2  # the visual columns of every row, once
+        importance = {"us": round(imp_us, 1), "shape": "B 1, H 32, Q = K 3392, visual 35..2914, r 576, bf16",
+                      "bytes": imp_bytes, "GBps": round(imp_bytes / (imp_us * 1e-6) / 1e9, 1), "launches": 3}
+        del imp_in
+
     ab, gb = attn_bytes(w), argmax_bytes(w)
     attn_avg_ms = sum(attn_ms) / K
     tail_avg_ms = sum(tail_ms) / K
@@ -416,6 +451,9 @@ def run_dreams(args, rank, world, local):
         kernels["verify_step_sampled"] = sampled
     if lm_head is not None:
         kernels["lm_head_argmax"] = lm_head
+    if importance is not None:
+        importance["frac_measured_hbm"] = round(importance["GBps"] / peak, 4)
+        kernels["visual_importance"] = importance
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -287,6 +287,27 @@ dreams_status_t dreams_lm_head_argmax(const void *hidden, int64_t rows, int64_t 
                                       int32_t *status_word, dreams_stream_t stream);
 
 /*
+ * Visual-token importance and top-r selection (Sec. 3.2 "Visual Token
+ * Compression", Eq. 2). attn: the target's final-layer prefill attention
+ * weights, [B, H, Q, K] contiguous, f32 or bf16. The visual tokens are key
+ * positions v0 .. v0 + n_vis - 1. For each sequence b:
+ *     importance[b][j] = 1 / (H Q) * sum_h sum_i attn[b][h][i][v0 + j]
+ *     keep[b][0..r)    = the positions v0 + j of the r largest importances
+ *                        (equal values: the lower position first), in
+ *                        increasing order
+ * Sums are f32, in a fixed order (the result does not depend on scheduling).
+ * 1 <= r <= n_vis <= 49152. Three launches: partial column sums over row
+ * ranges (HBM-bound), their sum in a fixed tree, then one CTA per sequence
+ * that selects. The workspace holds the partial sums and no state between
+ * calls.
+ */
+size_t dreams_visual_importance_workspace_size(int64_t B, int64_t H, int64_t Q, int64_t n_vis);
+dreams_status_t dreams_visual_importance(const void *attn, dreams_dtype_t dtype, int64_t B, int64_t H, int64_t Q,
+                                         int64_t K, int64_t v0, int64_t n_vis, int32_t r, float *importance,
+                                         int32_t *keep, void *workspace, size_t workspace_bytes,
+                                         dreams_stream_t stream);
+
+/*
  * Row-wise argmax for callers that cannot allocate device memory. The paper
  * has no counterpart to this call; it exists for integration. Some callers
  * cannot allocate, or cannot hand out a workspace, when the argmax runs: a

@@ -23,6 +23,10 @@ paper passage its C routine follows:
 * :func:`lm_head_argmax` -- the target's greedy prediction from its final
   hidden states: argmax over the vocabulary of H W^T, in fp64 (numpy's matmul
   as the product step), the same total order as :func:`argmax`.
+* :func:`visual_importance` -- the importance of each visual token, the mean of
+  its column of the final-layer attention over heads and queries, and the r
+  most important tokens kept (Sec. 3.2 "Visual Token Compression", Eq. 2);
+  :func:`top_r` is the selection alone.
 * :func:`accept_path` -- sequential acceptance with the target's token
   replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
 * :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
@@ -209,6 +213,38 @@ def lm_head_argmax(hidden_bits, weight_bits):
 def _bf16_to_f64(bits):
     b = np.ascontiguousarray(bits, dtype=np.uint16)
     return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def top_r(values, r: int, v0: int = 0) -> np.ndarray:
+    """Positions v0 + j of the r largest values per row (equal values: the
+    lower position first; NaN above every number), in increasing order."""
+    x = np.asarray(values)
+    B, n = x.shape
+    out = np.empty((B, r), np.int32)
+    for b in range(B):
+        row = x[b]
+        nan = np.isnan(row)
+        key = np.where(nan, np.inf, row)
+        order = np.lexsort((np.arange(n), -key, ~nan))  # NaN first, then larger, then lower position
+        out[b] = np.sort(order[:r]) + v0
+    return out
+
+
+def visual_importance(attn, v0: int, n_vis: int, r: int, bf16_bits: bool = False):
+    """(importance [B, n_vis] float64, keep [B, r]) from attention weights
+    [B, H, Q, K] (float32, or uint16 bf16 patterns): I_j = the sum over heads
+    and queries of A[:, :, :, v0 + j] divided by H Q (Eq. 2), summed head by
+    head in float64; keep = the r largest, positions in increasing order."""
+    a = np.asarray(attn)
+    B, H, Q, K = a.shape
+    imp = np.zeros((B, n_vis), np.float64)
+    for b in range(B):
+        for h in range(H):
+            blk = a[b, h, :, v0:v0 + n_vis]
+            blk = _bf16_to_f64(blk) if bf16_bits else blk.astype(np.float64)
+            imp[b] += blk.sum(axis=0)
+    imp /= float(H * Q)
+    return imp, top_r(imp, r, v0)
 
 
 def accept_path(am, parent, tokens, tree_len, kv_len, max_path: int):

@@ -88,6 +88,9 @@ def _lib() -> ctypes.CDLL:
                     "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
                     "dreams_lm_head_argmax_workspace_size": (sz, [i64]),
                     "dreams_lm_head_argmax": (ctypes.c_int, [p, i64, i64, i64, p, i64, i64, p, p, p, sz, p, p]),
+                    "dreams_visual_importance_workspace_size": (sz, [i64, i64, i64, i64]),
+                    "dreams_visual_importance": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, i64, i64, i64, i32,
+                                                                p, p, p, sz, p]),
                     "dreams_vocab_sample_workspace_size": (sz, [i64, i64]),
                     "dreams_vocab_sample": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, f32, p, p, p, sz, p]),
                     "dreams_verify_step_sampled_workspace_size": (sz, [ptr, i64]),
@@ -362,6 +365,28 @@ def lm_head_argmax(hidden: torch.Tensor, weight: torch.Tensor, out: Optional[tor
                                       0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
     _check("dreams_lm_head_argmax", st)
     return (out, out_max) if want_max or out_max is not None else out
+
+
+def visual_importance(attn: torch.Tensor, v0: int, n_vis: int, r: int, workspace: Optional[torch.Tensor] = None,
+                      stream=None):
+    """Eq. 2 importance of the visual tokens (key positions v0 .. v0+n_vis-1)
+    from attention weights [B, H, Q, K] (f32 / bf16, contiguous), and the r
+    kept positions in increasing order. Returns (importance f32 [B, n_vis],
+    keep int32 [B, r])."""
+    if attn.dtype not in (torch.float32, torch.bfloat16) or attn.dim() != 4 or not attn.is_contiguous():
+        raise TypeError("attn must be a contiguous [B, H, Q, K] float32/bfloat16 tensor")
+    B, H, Q, K = (int(x) for x in attn.shape)
+    dev = attn.device
+    imp = torch.empty((B, n_vis), dtype=torch.float32, device=dev)
+    keep = torch.empty((B, r), dtype=torch.int32, device=dev)
+    need = int(_lib().dreams_visual_importance_workspace_size(B, H, Q, n_vis))
+    if workspace is None:
+        workspace = _workspace("importance", need, dev, stream)
+    st = _lib().dreams_visual_importance(_ptr(attn), F32 if attn.dtype == torch.float32 else BF16, B, H, Q, K, v0,
+                                         n_vis, r, _ptr(imp), _ptr(keep), _ptr(workspace),
+                                         0 if workspace is None else workspace.numel(), _stream(stream))
+    _check("dreams_visual_importance", st)
+    return imp, keep
 
 
 def _walk_outputs(B: int, max_path: int, dev):
