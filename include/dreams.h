@@ -146,6 +146,35 @@ dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *
                                         int32_t *status_word, dreams_stream_t stream);
 
 /*
+ * Attention without a tree: the draft's cross-attention to target features,
+ * and the prefill self-attention of a target layer, optionally with each query
+ * row's attention entropy.
+ *   DREAMS_ATTN_FULL   query t of sequence b attends slots 0 .. kv_len[b] - 1:
+ *                      the cross-attention through which the draft reads the
+ *                      target's features S^l' (keys and values) with its own
+ *                      intermediate features E^j as queries (Sec. 3.2,
+ *                      "Adaptive Target Feature Injection");
+ *   DREAMS_ATTN_CAUSAL query t attends slots 0 .. kv_len[b] + t: its own slot
+ *                      is kv_len[b] + t (prefill of a layer, A = softmax(QK^T /
+ *                      sqrt(z)) of Sec. 3.3).
+ * q, out: bf16 [B, T_max, Hq, D]; q_len[b] in [1, T_max] query rows are
+ * computed (T_max <= 2^20); kv as for dreams_tree_verify_attn (FULL needs
+ * kv_len >= 1, CAUSAL kv_len + q_len <= capacity). lse and entropy: f32
+ * [B, T_max, Hq] or NULL. entropy[b][t][h] = -sum_j a_j ln a_j over the row's
+ * attention weights a (nats); the average over rows and heads is AE(l) of
+ * Sec. 3.3 (Adaptive Intermediate Feature Distillation). Accumulation as in
+ * dreams_tree_verify_attn; the entropy adds one f32 sum per row.
+ */
+#define DREAMS_ATTN_FULL 1
+#define DREAMS_ATTN_CAUSAL 2
+size_t dreams_attention_workspace_size(const dreams_kv_cache_t *kv, int32_t B, int32_t T_max, int32_t Hq,
+                                       int32_t mode, int32_t want_entropy);
+dreams_status_t dreams_attention(const void *q, const dreams_kv_cache_t *kv, int32_t layer, const int32_t *q_len,
+                                 const int32_t *kv_len, int32_t B, int32_t T_max, int32_t Hq, float scale,
+                                 int32_t mode, void *out, float *lse, float *entropy, void *workspace,
+                                 size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream);
+
+/*
  * Row-wise argmax (the target's greedy prediction, Sec. 2 "Speculative
  * decoding" at temperature 0): out_idx[r] = argmax_v logits[r * row_stride + v]
  * for v < V, under the total order "greater value wins, equal values (+0 ==

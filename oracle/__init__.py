@@ -27,6 +27,11 @@ paper passage its C routine follows:
   its column of the final-layer attention over heads and queries, and the r
   most important tokens kept (Sec. 3.2 "Visual Token Compression", Eq. 2);
   :func:`top_r` is the selection alone.
+* :func:`attention_rows` -- attention without a tree: the draft's cross-attention
+  to the target's features (every query sees slots 0 .. L-1; Sec. 3.2, "Adaptive
+  Target Feature Injection") or a layer's causal prefill (query t sees slots
+  0 .. L+t), with each row's attention entropy -sum_j a_j ln a_j, whose mean
+  over rows and heads is AE(l) (Sec. 3.3).
 * :func:`accept_path` -- sequential acceptance with the target's token
   replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
 * :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
@@ -245,6 +250,34 @@ def visual_importance(attn, v0: int, n_vis: int, r: int, bf16_bits: bool = False
             imp[b] += blk.sum(axis=0)
     imp /= float(H * Q)
     return imp, top_r(imp, r, v0)
+
+
+def attention_rows(q, k, v, q_len, kv_len, scale: float, causal: bool, sel):
+    """(out [n, D], lse [n], entropy [n]) in float64 for the selected (b, t, h)
+    triples. q: float [B, T_max, Hq, D]; k, v: float [B, capacity, Hkv, D]
+    (contiguous caches). Row (b, t, h) attends slots 0 .. kv_len[b] - 1
+    (causal=False) or 0 .. kv_len[b] + t (causal=True) of KV head h // G:
+        s_j = scale <q, K_j>, m = max s, w_j = exp(s_j - m), Z = sum w,
+        out = sum w_j V_j / Z, lse = m + ln Z, entropy = -sum (w/Z) ln(w/Z)."""
+    q = np.asarray(q, np.float64)
+    k = np.asarray(k, np.float64)
+    v = np.asarray(v, np.float64)
+    Hq, Hkv = q.shape[2], k.shape[2]
+    G = Hq // Hkv
+    outs, lses, ents = [], [], []
+    for b, t, h in sel:
+        n = int(kv_len[b]) + (int(t) + 1 if causal else 0)
+        g = h // G
+        s = scale * (k[b, :n, g, :] @ q[b, t, h, :])
+        m = s.max()
+        w = np.exp(s - m)
+        Z = w.sum()
+        a = w / Z
+        outs.append((a[:, None] * v[b, :n, g, :]).sum(axis=0))
+        lses.append(m + np.log(Z))
+        nz = a > 0
+        ents.append(-(a[nz] * np.log(a[nz])).sum())
+    return np.array(outs), np.array(lses), np.array(ents)
 
 
 def accept_path(am, parent, tokens, tree_len, kv_len, max_path: int):

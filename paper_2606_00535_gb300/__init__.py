@@ -86,6 +86,9 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, p, p, p, p,
                                                           p, p, sz, p, p]),
                     "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
+                    "dreams_attention_workspace_size": (sz, [pkv, i32, i32, i32, i32, i32]),
+                    "dreams_attention": (ctypes.c_int, [p, pkv, i32, p, p, i32, i32, i32, f32, i32, p, p, p, p, sz,
+                                                        p, p]),
                     "dreams_lm_head_argmax_workspace_size": (sz, [i64]),
                     "dreams_lm_head_argmax": (ctypes.c_int, [p, i64, i64, i64, p, i64, i64, p, p, p, sz, p, p]),
                     "dreams_visual_importance_workspace_size": (sz, [i64, i64, i64, i64]),
@@ -333,6 +336,37 @@ def vocab_sample(logits: torch.Tensor, temperature: float, uniforms: torch.Tenso
         _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
     _check("dreams_vocab_sample", st)
     return out
+
+
+ATTN_FULL = 1    # query t attends slots 0 .. kv_len - 1 (cross-attention)
+ATTN_CAUSAL = 2  # query t attends slots 0 .. kv_len + t (prefill self-attention)
+
+
+def attention(q: torch.Tensor, kv: KVCache, q_len: torch.Tensor, kv_len: torch.Tensor, scale: float, mode: int,
+              layer: int = 0, out: Optional[torch.Tensor] = None, want_lse: bool = False,
+              want_entropy: bool = False, workspace: Optional[torch.Tensor] = None,
+              status: Optional[torch.Tensor] = None, stream=None):
+    """Attention without a tree (ATTN_FULL: the draft's cross-attention to
+    target features; ATTN_CAUSAL: a layer's prefill). q: bf16 [B, T_max, Hq,
+    D]. Returns (out, lse, entropy); lse and entropy are None unless asked."""
+    dev = q.device
+    _need(q, "q", torch.bfloat16, dev)
+    for n, t in (("q_len", q_len), ("kv_len", kv_len)):
+        _need(t, n, torch.int32, dev)
+    B, T_max, Hq = int(q.shape[0]), int(q.shape[1]), int(q.shape[2])
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, dev)
+    lse = torch.empty((B, T_max, Hq), dtype=torch.float32, device=dev) if want_lse else None
+    ent = torch.empty((B, T_max, Hq), dtype=torch.float32, device=dev) if want_entropy else None
+    need = int(_lib().dreams_attention_workspace_size(ctypes.byref(kv._c), B, T_max, Hq, mode, int(want_entropy)))
+    if workspace is None:
+        workspace = _workspace("attention", need, dev, stream)
+    st = _lib().dreams_attention(_ptr(q), ctypes.byref(kv._c), layer, _ptr(q_len), _ptr(kv_len), B, T_max, Hq,
+                                 float(scale), mode, _ptr(out), _ptr(lse), _ptr(ent), _ptr(workspace),
+                                 0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
+    _check("dreams_attention", st)
+    return out, lse, ent
 
 
 def lm_head_argmax(hidden: torch.Tensor, weight: torch.Tensor, out: Optional[torch.Tensor] = None,

@@ -102,7 +102,18 @@ struct AttnParams {
   float2 *ws_ml;   // [B][Hkv][nrb][nsplit][ROWS] (max in log2 units, sum)
   int32_t *order;  // [B * nsplit] pair index b * nsplit + split, longest first; nullptr: natural order
   int32_t *status;
+  int32_t mode;    // ATTN_TREE, ATTN_FULL or ATTN_CAUSAL: which slots a query row attends
+  float *ent;      // [B, T_max, Hq] attention entropy of each query row (nats), with the entropy kernels
+  float *ws_w;     // [B][Hkv][nrb][nsplit][ROWS] sum_j P_j (x_j - m) of the split partials (entropy)
 };
+
+constexpr int ATTN_TREE = 0;    // prefix slots plus the node's own ancestors among the tree slots
+constexpr int ATTN_FULL = 1;    // slots 0 .. kv_len - 1 (cross-attention: no mask)
+constexpr int ATTN_CAUSAL = 2;  // slots 0 .. kv_len + t for query t (prefill self-attention)
+
+// Keys of sequence b: the prefix plus the query rows' own slots (tree,
+// causal), or the prefix alone (full).
+__device__ __forceinline__ int key_total(const AttnParams &p, int L, int T) { return p.mode == ATTN_FULL ? L : L + T; }
 
 struct TcParams {
   CUtensorMap tmap_q;
@@ -145,8 +156,9 @@ __device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
 __device__ __forceinline__ int split_tiles(const AttnParams &p, int b, int s) {
   const int T = __ldg(p.tree_len + b);
   const int L = __ldg(p.kv_len + b);
-  if (T < 1 || T > p.T_max || L < 0 || L > p.capacity - T) return 0;
-  const int tiles = (L + T + KT - 1) / KT;
+  const int total = key_total(p, L, T);
+  if (T < 1 || T > p.T_max || L < 0 || total > p.capacity || total < 1) return 0;
+  const int tiles = (total + KT - 1) / KT;
   const int ct = p.chunk / KT;
   return ::max(0, ::min(ct, tiles - s * ct));
 }
@@ -207,7 +219,7 @@ __global__ void __launch_bounds__(ORDER_THREADS) tree_attn_order_kernel(const At
   }
 }
 
-template <int D>
+template <int D, bool ENT>
 __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_constant__ TcParams P) {
   const AttnParams &p = P.a;
   constexpr int NR = D / 64;                     // 128-byte column regions of a row
@@ -231,7 +243,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const int per_pair = p.Hkv * p.nrb;
   const int pair_pos = blockIdx.x / per_pair;
   const int gr = blockIdx.x - pair_pos * per_pair;
-  const int g = gr / p.nrb, rb = gr - g * p.nrb;
+  const int g = gr / p.nrb, rb_raw = gr - g * p.nrb;
+  // causal rows: the last row blocks have the most keys, so they go first
+  const int rb = p.mode == ATTN_CAUSAL ? p.nrb - 1 - rb_raw : rb_raw;
   int pair = pair_pos;
   if (p.order != nullptr) {
     // the order comes from the preceding kernel (programmatic dependent launch)
@@ -246,14 +260,17 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_TREE_LEN);
     return;
   }
-  if (L < 0 || L > p.capacity - T) {
+  const int total = key_total(p, L, T);
+  if (L < 0 || total > p.capacity || total < 1) {
     if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_KV_LEN);
     return;
   }
-  const int total = L + T;
   const int nsplit_b = (total + p.chunk - 1) / p.chunk;
   const int t0 = rb * p.TB;  // first tree node of the row block
   if (split >= nsplit_b || t0 >= T) return;
+  // keys any row of the block may attend: a causal block stops after its last row's own slot
+  const int kend = p.mode == ATTN_CAUSAL ? L + ::min(T, t0 + p.TB) : total;
+  if (split * p.chunk >= kend) return;
   const int rows_blk = ::min(p.TB, T - t0) * p.G;  // real query rows of this CTA
   // softmax warps whose 32 rows hold at least one real query row
   const int n_act = ::min(4, (rows_blk + 31) / 32);
@@ -296,7 +313,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const uint32_t tmem = s_tmem;
 
   const int c0 = split * p.chunk;
-  const int c1 = ::min(c0 + p.chunk, total);
+  const int c1 = ::min(c0 + p.chunk, kend);
   const int ntiles = (c1 - c0 + KT - 1) / KT;
   volatile int *abort_flag = &s_abort;
   // abort codes: 1 = a wait timed out, 2 = malformed tree (nothing to compute)
@@ -314,7 +331,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const int row = 32 * (warp & 3) + lane;    // TMEM lane = query row
   const bool real_row = row < rows_blk;
   const int t_row = t0 + row / p.G;
-  if (warp == MMA_WARP) {
+  if (warp == MMA_WARP && p.mode != ATTN_TREE) {
+    if (lane == 0) s_flag = 0;  // no tree: every key set is a prefix of the slots
+    named_sync(2, 288);
+  } else if (warp == MMA_WARP) {
     int par[2], bad = 0;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -365,6 +385,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const bool tree_ok = (warp == TMA_WARP) || !s_flag;
 
   float m_ref = -INFINITY, l = 0.f;  // this thread's row state (softmax warps)
+  float wsum = 0.f;                  // entropy: sum_j P_j (x_j - m_ref), x = scaled score in log2 units
   bool sm_ok = false;                // the softmax loop ran to completion
 
   if (warp == TMA_WARP) {
@@ -512,7 +533,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   } else if ((warp & 3) < n_act && tree_ok) {
     // ---------------- softmax warpgroup wg: tiles wg, wg + 2, ...
     const uint32_t tl = tmem + (uint32_t(32 * (warp & 3)) << 16) + 256u * wg;
-    const unsigned long long anc = real_row ? s_anc[t_row] : 0ull;
+    const unsigned long long anc = (real_row && p.mode == ATTN_TREE) ? s_anc[t_row] : 0ull;
+    // slots below lim are allowed besides the ancestors: the prefix, or for a
+    // causal row the prefix and the rows up to its own
+    const int lim = p.mode == ATTN_CAUSAL ? L + t_row + 1 : L;
     const int nw = (ntiles - wg + 1) / 2;
     bool ok = true;
     for (int ii = 0; ii < nw; ++ii) {
@@ -531,7 +555,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         tc::tmem_ld32(tl + 32 * q4, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * q4]));
       tc::tmem_wait_ld();
       const int s0 = c0 + j * KT;
-      if ((s0 + KT > L) || (s0 + KT > c1)) {
+      if ((s0 + KT > lim) || (s0 + KT > c1)) {
         // tree columns outside the row's ancestors, and columns past this
         // split: -inf. The allowed columns as four 32-bit words: prefix
         // slots (< L), the row's ancestors among the tree slots (bit a of
@@ -542,7 +566,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
 #pragma unroll
         for (int q = 0; q < KT / 32; ++q) {
           const int cb = s0 + 32 * q;  // slot of bit 0 of this word
-          const int np = L - cb, ne = c1 - cb, sh = cb - L;
+          const int np = lim - cb, ne = c1 - cb, sh = cb - L;
           const uint32_t pre = np >= 32 ? 0xffffffffu : (np <= 0 ? 0u : (1u << np) - 1u);
           const uint32_t end = ne >= 32 ? 0xffffffffu : (ne <= 0 ? 0u : (1u << ne) - 1u);
           const uint32_t tr = (sh >= 64 || sh <= -32) ? 0u
@@ -569,7 +593,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const bool resc = mx > m_ref + RESCALE;
       float corr = 1.f;
       if (resc) {
-        corr = (m_ref == -INFINITY) ? 0.f : tc::ex2(m_ref - mx);
+        const float m_old = m_ref;
+        corr = (m_old == -INFINITY) ? 0.f : tc::ex2(m_old - mx);
+        // the entropy sum sum_j P_j (x_j - m) follows the new reference
+        if (ENT) wsum = (m_old == -INFINITY) ? 0.f : corr * (wsum - (mx - m_old) * l);
         m_ref = mx;
         l *= corr;
       }
@@ -578,6 +605,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       // time (f32x2 add), P as bf16 pairs
       const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2), nmu2 = f32x2(nmu, nmu);
       uint64_t acc2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
+      uint64_t wacc2 = f32x2(0.f, 0.f);  // entropy: sum of P e over the tile
 #pragma unroll
       for (int q4 = 0; q4 < KT / 32; ++q4) {
         uint32_t pk[16];
@@ -589,6 +617,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
                       e0, e1);
           const float p0 = tc::ex2(e0), p1 = tc::ex2(e1);
           acc2[c & 1] = fadd2(acc2[c & 1], f32x2(p0, p1));
+          // masked slots have e = -inf and P = 0: clamp e so that P e is 0, not NaN
+          if (ENT) wacc2 = ffma2(f32x2(p0, p1), f32x2(fmaxf(e0, -200.f), fmaxf(e1, -200.f)), wacc2);
           pk[c] = pack_bf16x2(p0, p1);
         }
         tc::tmem_st16(tl + 16 * q4, pk);  // P (bf16 pairs) over the first 64 columns of S
@@ -598,6 +628,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         f32x2_split(acc2[0], a0, a1);
         f32x2_split(acc2[1], b0, b1);
         l += (a0 + a1) + (b0 + b1);
+        if (ENT) {
+          f32x2_split(wacc2, a0, a1);
+          wsum += a0 + a1;
+        }
       }
       if (c1 - s0 < KT) {
         // slots past the sequence end may hold any bits (0 * NaN = NaN in the
@@ -647,9 +681,14 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   // copy takes the Q region and the K ring, (m, l) the last V stage.
   if (warp < 8) {
     const bool act = (warp & 3) < n_act && tree_ok;
-    const bool direct = nsplit_b == 1;
+    // the output directly, unless the block's keys span several splits
+    const bool direct = (kend + p.chunk - 1) / p.chunk == 1;
     float2 *s_ml = reinterpret_cast<float2 *>(smem + Q_BYTES + (NK + NV - 1) * KV_TILE);
-    if (act && sm_ok) s_ml[wg * ROWS + row] = make_float2(m_ref, l);
+    float *s_w = reinterpret_cast<float *>(s_ml + 2 * ROWS);  // entropy sums of both warpgroups
+    if (act && sm_ok) {
+      s_ml[wg * ROWS + row] = make_float2(m_ref, l);
+      if (ENT) s_w[wg * ROWS + row] = wsum;
+    }
     tc::fence_before_sync();
     named_sync(1, 256);
     tc::fence_after_sync();
@@ -701,13 +740,21 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         }
       }
       if (wg == 0 && real_row) {
+        // entropy of the row: with P_j = 2^(x_j - M) and Z = sum_j P_j,
+        // H = ln Z - ln 2 * sum_j P_j (x_j - M) / Z; each warpgroup's sum moves
+        // from its own reference m to M as c * (W + (m - M) l)
+        float Wt = 0.f;
+        if (ENT) {
+          if (ca != 0.f) Wt += ca * (s_w[row] + (a.x - M) * a.y);
+          if (cb != 0.f) Wt += cb * (s_w[ROWS + row] + (c.x - M) * c.y);
+        }
+        const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + (row - (t_row - t0) * p.G);
         if (direct) {
-          if (p.lse != nullptr) {
-            const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + (row - (t_row - t0) * p.G);
-            p.lse[orow] = (M + log2f(Ls)) * LN2;
-          }
+          if (p.lse != nullptr) p.lse[orow] = (M + log2f(Ls)) * LN2;
+          if (ENT && p.ent != nullptr) p.ent[orow] = logf(Ls) - LN2 * Wt / Ls;
         } else {
           p.ws_ml[slot + row] = make_float2(Ls > 0.f ? M : -INFINITY, Ls);
+          if (ENT) p.ws_w[slot + row] = Ls > 0.f ? Wt : 0.f;
         }
       }
     }
@@ -758,7 +805,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
 // key wrote zeros), so a row costs about one memory latency. Launched as a
 // programmatic dependent of the attention kernel: griddepcontrol.wait returns
 // once that grid has completed and its writes are visible.
-template <int D>
+template <int D, bool ENT>
 __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   constexpr int NL = D / 4;  // lanes holding 4 columns each
@@ -773,10 +820,17 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
   if (b >= p.B) return;
   const int T = __ldg(p.tree_len + b);
   const int L = __ldg(p.kv_len + b);
-  if (T < 1 || T > p.T_max || L < 0 || L > p.capacity - T) return;
-  const int nsplit_b = (L + T + p.chunk - 1) / p.chunk;
+  const int total = key_total(p, L, T);
+  if (T < 1 || T > p.T_max || L < 0 || total > p.capacity || total < 1) return;
   const int t0 = rb * p.TB;
-  if (nsplit_b == 1 || t0 >= T || r >= ::min(p.TB, T - t0) * p.G) return;
+  if (t0 >= T || r >= ::min(p.TB, T - t0) * p.G) return;
+  // splits of the row block (it was written directly when there is one) and
+  // of this row (a causal row's keys end at its own slot)
+  const int kend = p.mode == ATTN_CAUSAL ? L + ::min(T, t0 + p.TB) : total;
+  const int nsplit_blk = (kend + p.chunk - 1) / p.chunk;
+  if (nsplit_blk == 1) return;
+  const int tn = r / p.G;
+  const int nsplit_b = p.mode == ATTN_CAUSAL ? (L + t0 + tn + 1 + p.chunk - 1) / p.chunk : nsplit_blk;
 
   const int64_t sbase = item * p.nsplit * ROWS + r;
   float4 x[8];
@@ -786,10 +840,13 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
                ? __ldcg(reinterpret_cast<const float4 *>(p.ws_o + (sbase + int64_t(k) * ROWS) * D) + lane)
                : make_float4(0.f, 0.f, 0.f, 0.f);
   const float2 ml = lane < nsplit_b ? __ldcg(p.ws_ml + sbase + int64_t(lane) * ROWS) : make_float2(-INFINITY, 0.f);
+  const float wl = (ENT && lane < nsplit_b) ? __ldcg(p.ws_w + sbase + int64_t(lane) * ROWS) : 0.f;
   int bad = 0;  // the attention kernel skipped malformed trees; so does the merge
-  for (int i = lane; i < T; i += 32) {
-    const int par = __ldg(p.parent + int64_t(b) * p.T_max + i);
-    bad |= (i == 0) ? (par != -1) : (par < 0 || par >= i);
+  if (p.mode == ATTN_TREE) {
+    for (int i = lane; i < T; i += 32) {
+      const int par = __ldg(p.parent + int64_t(b) * p.T_max + i);
+      bad |= (i == 0) ? (par != -1) : (par < 0 || par >= i);
+    }
   }
   if (__any_sync(0xffffffffu, bad)) return;
 
@@ -798,8 +855,12 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
   for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
   const float w = ml.y > 0.f ? tc::ex2(ml.x - M) : 0.f;
   float Ls = w * ml.y;
+  float Wt = (ENT && ml.y > 0.f) ? w * (wl + (ml.x - M) * ml.y) : 0.f;
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
+  for (int off = 16; off > 0; off >>= 1) {
+    Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
+    if (ENT) Wt += __shfl_xor_sync(0xffffffffu, Wt, off);
+  }
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
@@ -821,13 +882,15 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
   }
   if (lane >= NL) return;
   const float inv = 1.f / Ls;
-  const int tn = r / p.G;
   const int64_t orow = (int64_t(b) * p.T_max + t0 + tn) * p.Hq + g * p.G + (r - tn * p.G);
   uint2 pk;
   pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
   pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
   *reinterpret_cast<uint2 *>(p.out + orow * D + lane * 4) = pk;
-  if (p.lse != nullptr && lane == 0) p.lse[orow] = (M + log2f(Ls)) * LN2;
+  if (lane == 0) {
+    if (p.lse != nullptr) p.lse[orow] = (M + log2f(Ls)) * LN2;
+    if (ENT && p.ent != nullptr) p.ent[orow] = logf(Ls) - LN2 * Wt / Ls;
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -837,7 +900,7 @@ struct AttnPlan {
   int nsplit;
   int chunk;
   bool ordered;
-  size_t ws_o_bytes, ws_ml_bytes, order_bytes;
+  size_t ws_o_bytes, ws_ml_bytes, ws_w_bytes, order_bytes;
   size_t ws_bytes;
 };
 
@@ -848,12 +911,12 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // chunk plus a fixed start-up and write-out of about four tiles: the first
 // tiles of all SMs arrive together; a merge pass about two more); splits of
 // >= 256 tokens, at most MAX_SPLITS.
-AttnPlan plan(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
+AttnPlan plan(const dreams_kv_cache_t *kv, int B, int T_max, int Hq, bool ent) {
   AttnPlan pl{};
   const int G = Hq / kv->Hkv;
   pl.TB = std::max(1, ROWS / G);
-  pl.nrb = (tree->T_max + pl.TB - 1) / pl.TB;
-  const int64_t base = int64_t(tree->B) * kv->Hkv * pl.nrb;
+  pl.nrb = (T_max + pl.TB - 1) / pl.TB;
+  const int64_t base = int64_t(B) * kv->Hkv * pl.nrb;
   const int64_t sms = num_sms();
   const int64_t max_ns = std::max<int64_t>(1, (kv->capacity + 255) / 256);
   int64_t best_ns = 1;
@@ -877,17 +940,19 @@ AttnPlan plan(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
     const size_t slots = size_t(base) * pl.nsplit * ROWS;
     pl.ws_o_bytes = align_up(slots * kv->D * sizeof(float), 256);
     pl.ws_ml_bytes = align_up(slots * sizeof(float2), 256);
+    if (ent) pl.ws_w_bytes = align_up(slots * sizeof(float), 256);
   }
-  pl.ordered = tree->B > 1;
-  if (pl.ordered) pl.order_bytes = align_up(size_t(tree->B) * pl.nsplit * sizeof(int32_t), 256);
-  pl.ws_bytes = pl.ws_o_bytes + pl.ws_ml_bytes + pl.order_bytes;
+  pl.ordered = B > 1;
+  if (pl.ordered) pl.order_bytes = align_up(size_t(B) * pl.nsplit * sizeof(int32_t), 256);
+  pl.ws_bytes = pl.ws_o_bytes + pl.ws_ml_bytes + pl.ws_w_bytes + pl.order_bytes;
   return pl;
 }
 
-bool valid_shapes(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int Hq) {
-  return kv != nullptr && tree != nullptr && tree->B >= 1 && tree->B <= 65535 && tree->T_max >= 1 &&
-         tree->T_max <= 64 && kv->Hkv >= 1 && kv->Hkv <= 65535 && Hq >= kv->Hkv && Hq % kv->Hkv == 0 &&
-         Hq / kv->Hkv <= ROWS && kv->capacity >= 1 && kv->n_layers >= 1;
+bool valid_shapes(const dreams_kv_cache_t *kv, int B, int T_max, int Hq, int mode) {
+  const int tmax_limit = mode == ATTN_TREE ? 64 : (1 << 20);
+  return kv != nullptr && B >= 1 && B <= 65535 && T_max >= 1 && T_max <= tmax_limit && kv->Hkv >= 1 &&
+         kv->Hkv <= 65535 && Hq >= kv->Hkv && Hq % kv->Hkv == 0 && Hq / kv->Hkv <= ROWS && kv->capacity >= 1 &&
+         kv->n_layers >= 1;
 }
 
 // 4-D view of one layer's K or V cache with a (64 columns, 1 head, 64 slots,
@@ -954,7 +1019,7 @@ cudaError_t launch_pdl(const void *func, dim3 grid, dim3 block, size_t smem, cud
   return cudaLaunchKernelExC(&cfg, func, args);
 }
 
-template <int D>
+template <int D, bool ENT>
 dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_cache_t *kv, const void *k,
                        const void *v, int B, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<D>();
@@ -963,7 +1028,7 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   cudaGetDevice(&dev);
   if (dev < 31 && !(configured_mask & (1 << dev))) {
     cudaError_t e =
-        cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        cudaFuncSetAttribute(tree_attn_tc_kernel<D, ENT>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e != cudaSuccess) {
       set_last_cuda_error(e);
       return DREAMS_ERR_CUDA;
@@ -984,7 +1049,7 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   }
   const int64_t ctas = int64_t(B) * pl.nsplit * a.Hkv * pl.nrb;
   void *args_attn[] = {&P};
-  cudaError_t e = launch_pdl(reinterpret_cast<const void *>(tree_attn_tc_kernel<D>), dim3(unsigned(ctas)),
+  cudaError_t e = launch_pdl(reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT>), dim3(unsigned(ctas)),
                              dim3(THREADS), smem, stream, pl.ordered, args_attn);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
@@ -995,7 +1060,7 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   const int64_t rows = int64_t(B) * a.Hkv * pl.nrb * ROWS;
   AttnParams am = a;
   void *args_merge[] = {&am};
-  e = launch_pdl(reinterpret_cast<const void *>(tree_attn_merge_kernel<D>), dim3(unsigned((rows + 7) / 8)),
+  e = launch_pdl(reinterpret_cast<const void *>(tree_attn_merge_kernel<D, ENT>), dim3(unsigned((rows + 7) / 8)),
                  dim3(256), 0, stream, true, args_merge);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
@@ -1009,33 +1074,22 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
 
 using namespace dreams;
 
-extern "C" size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv,
-                                                         const dreams_tree_t *tree, int32_t Hq) {
-  if (!valid_shapes(kv, tree, Hq)) return 0;
-  return plan(kv, tree, Hq).ws_bytes;
-}
+namespace {
 
-extern "C" int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
-                                                    int32_t Hq) {
-  if (!valid_shapes(kv, tree, Hq) || (kv->D != 64 && kv->D != 128)) return 0;
-  const AttnPlan pl = plan(kv, tree, Hq);
-  return 1 + (pl.ordered ? 1 : 0) + (pl.nsplit > 1 ? 1 : 0);
-}
-
-extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
-                                                   const dreams_tree_t *tree, int32_t Hq, float scale,
-                                                   void *out, float *lse, void *workspace,
-                                                   size_t workspace_bytes, int32_t *status_word,
-                                                   dreams_stream_t stream) {
-  if (q == nullptr || out == nullptr || kv == nullptr || tree == nullptr) return DREAMS_ERR_INVALID_ARG;
-  if (kv->k == nullptr || kv->v == nullptr || tree->parent == nullptr || tree->tree_len == nullptr ||
-      tree->kv_len == nullptr)
+// The shared body of the two attention entry points.
+dreams_status_t attention_impl(const void *q, const dreams_kv_cache_t *kv, int32_t layer, const int32_t *parent,
+                               const int32_t *q_len, const int32_t *kv_len, int32_t B, int32_t T_max, int32_t Hq,
+                               float scale, int32_t mode, void *out, float *lse, float *ent, void *workspace,
+                               size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream) {
+  if (q == nullptr || out == nullptr || kv == nullptr || q_len == nullptr || kv_len == nullptr)
     return DREAMS_ERR_INVALID_ARG;
-  if (!valid_shapes(kv, tree, Hq)) return DREAMS_ERR_INVALID_ARG;
+  if (kv->k == nullptr || kv->v == nullptr || (mode == ATTN_TREE && parent == nullptr)) return DREAMS_ERR_INVALID_ARG;
+  if (!valid_shapes(kv, B, T_max, Hq, mode)) return DREAMS_ERR_INVALID_ARG;
   if (kv->D != 64 && kv->D != 128) return DREAMS_ERR_UNSUPPORTED;
   if (layer < 0 || layer >= kv->n_layers || kv->layer_stride < 0) return DREAMS_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out) || !aligned16(kv->k) || !aligned16(kv->v) ||
-      (kv->layer_stride * 2) % 16 != 0 || (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3)))
+      (kv->layer_stride * 2) % 16 != 0 || (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3)) ||
+      (ent != nullptr && (reinterpret_cast<uintptr_t>(ent) & 3)))
     return DREAMS_ERR_INVALID_ARG;
   if (!isfinite(scale) || !(scale > 0.f)) return DREAMS_ERR_INVALID_ARG;
   if (kv->page_table != nullptr) {
@@ -1043,10 +1097,13 @@ extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_k
     if (kv->pages_per_seq < 1 || kv->num_pages < 1 || int64_t(kv->pages_per_seq) * 64 != kv->capacity)
       return DREAMS_ERR_INVALID_ARG;
   }
-  const AttnPlan pl = plan(kv, tree, Hq);
+  const bool want_ent = ent != nullptr;
+  const AttnPlan pl = plan(kv, B, T_max, Hq, want_ent);
   if (pl.ws_bytes > 0 && (workspace == nullptr || workspace_bytes < pl.ws_bytes || !aligned16(workspace)))
     return DREAMS_ERR_WORKSPACE;
-  if (int64_t(tree->B) * pl.nsplit * kv->Hkv * pl.nrb > 0x7fffffff) return DREAMS_ERR_UNSUPPORTED;
+  if (int64_t(B) * pl.nsplit * kv->Hkv * pl.nrb > 0x7fffffff ||
+      int64_t(B) * kv->Hkv * pl.nrb * ROWS / 8 > 0x7fffffff)
+    return DREAMS_ERR_UNSUPPORTED;
 
   AttnParams p{};
   p.q = static_cast<const __nv_bfloat16 *>(q);
@@ -1056,11 +1113,11 @@ extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_k
   p.pages_per_seq = kv->pages_per_seq;
   p.num_pages = kv->num_pages;
   p.capacity = kv->capacity;
-  p.parent = tree->parent;
-  p.tree_len = tree->tree_len;
-  p.kv_len = tree->kv_len;
-  p.B = tree->B;
-  p.T_max = tree->T_max;
+  p.parent = parent;
+  p.tree_len = q_len;
+  p.kv_len = kv_len;
+  p.B = B;
+  p.T_max = T_max;
   p.Hq = Hq;
   p.Hkv = kv->Hkv;
   p.G = Hq / kv->Hkv;
@@ -1069,15 +1126,62 @@ extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_k
   p.nsplit = pl.nsplit;
   p.chunk = pl.chunk;
   p.scale_log2 = scale * LOG2E;
+  p.mode = mode;
+  p.ent = ent;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   if (pl.nsplit > 1) {
     p.ws_o = reinterpret_cast<float *>(ws);
     p.ws_ml = reinterpret_cast<float2 *>(ws + pl.ws_o_bytes);
+    if (want_ent) p.ws_w = reinterpret_cast<float *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes);
   }
-  if (pl.ordered) p.order = reinterpret_cast<int32_t *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes);
+  if (pl.ordered) p.order = reinterpret_cast<int32_t *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes + pl.ws_w_bytes);
   p.status = status_word;
   const void *k = static_cast<const __nv_bfloat16 *>(kv->k) + int64_t(layer) * kv->layer_stride;
   const void *v = static_cast<const __nv_bfloat16 *>(kv->v) + int64_t(layer) * kv->layer_stride;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  return kv->D == 128 ? launch<128>(p, pl, kv, k, v, tree->B, s) : launch<64>(p, pl, kv, k, v, tree->B, s);
+  if (want_ent)
+    return kv->D == 128 ? launch<128, true>(p, pl, kv, k, v, B, s) : launch<64, true>(p, pl, kv, k, v, B, s);
+  return kv->D == 128 ? launch<128, false>(p, pl, kv, k, v, B, s) : launch<64, false>(p, pl, kv, k, v, B, s);
+}
+
+}  // namespace
+
+extern "C" size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv,
+                                                         const dreams_tree_t *tree, int32_t Hq) {
+  if (tree == nullptr || !valid_shapes(kv, tree->B, tree->T_max, Hq, ATTN_TREE)) return 0;
+  return plan(kv, tree->B, tree->T_max, Hq, false).ws_bytes;
+}
+
+extern "C" int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
+                                                    int32_t Hq) {
+  if (tree == nullptr || !valid_shapes(kv, tree->B, tree->T_max, Hq, ATTN_TREE) || (kv->D != 64 && kv->D != 128))
+    return 0;
+  const AttnPlan pl = plan(kv, tree->B, tree->T_max, Hq, false);
+  return 1 + (pl.ordered ? 1 : 0) + (pl.nsplit > 1 ? 1 : 0);
+}
+
+extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+                                                   const dreams_tree_t *tree, int32_t Hq, float scale,
+                                                   void *out, float *lse, void *workspace,
+                                                   size_t workspace_bytes, int32_t *status_word,
+                                                   dreams_stream_t stream) {
+  if (tree == nullptr) return DREAMS_ERR_INVALID_ARG;
+  return attention_impl(q, kv, layer, tree->parent, tree->tree_len, tree->kv_len, tree->B, tree->T_max, Hq, scale,
+                        ATTN_TREE, out, lse, nullptr, workspace, workspace_bytes, status_word, stream);
+}
+
+extern "C" size_t dreams_attention_workspace_size(const dreams_kv_cache_t *kv, int32_t B, int32_t T_max, int32_t Hq,
+                                                  int32_t mode, int32_t want_entropy) {
+  if ((mode != DREAMS_ATTN_FULL && mode != DREAMS_ATTN_CAUSAL) || !valid_shapes(kv, B, T_max, Hq, mode)) return 0;
+  return plan(kv, B, T_max, Hq, want_entropy != 0).ws_bytes;
+}
+
+extern "C" dreams_status_t dreams_attention(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+                                            const int32_t *q_len, const int32_t *kv_len, int32_t B, int32_t T_max,
+                                            int32_t Hq, float scale, int32_t mode, void *out, float *lse,
+                                            float *entropy, void *workspace, size_t workspace_bytes,
+                                            int32_t *status_word, dreams_stream_t stream) {
+  if (mode != DREAMS_ATTN_FULL && mode != DREAMS_ATTN_CAUSAL) return DREAMS_ERR_INVALID_ARG;
+  return attention_impl(q, kv, layer, nullptr, q_len, kv_len, B, T_max, Hq, scale, mode, out, lse, entropy,
+                        workspace, workspace_bytes, status_word, stream);
 }
