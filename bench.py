@@ -19,6 +19,7 @@ sample of the same workload per step and scales it to a full step.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
 import statistics
@@ -52,6 +53,8 @@ def parse():
                     help="skip the extra timing of the temperature-1 verification tail")
     ap.add_argument("--no-lm-head", action="store_true",
                     help="skip the extra timing of the LM head with the fused argmax")
+    ap.add_argument("--no-modes", action="store_true",
+                    help="skip the extra timings of the draft cross-attention and the entropy prefill")
     ap.add_argument("--no-importance", action="store_true",
                     help="skip the extra timing of the visual-token importance (Eq. 2) on a LLaVA-7B-shaped prefill")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
@@ -425,6 +428,70 @@ def run_dreams(args, rank, world, local):
                       "bytes": imp_bytes, "GBps": round(imp_bytes / (imp_us * 1e-6) / 1e9, 1), "launches": 3}
         del imp_in
 
+    # ---- attention without a tree, LLaVA-7B layer shapes (32 heads, D 128):
+    # the draft's cross-attention of 60 draft positions to the 3392 target
+    # features, and a layer's causal prefill of 3392 tokens with each row's
+    # entropy (the AE(l) of the distillation-layer choice)
+    modes = None
+    if not args.no_modes:
+        Hm, Dm, Nm, Tq = 32, 128, 3392, 60
+        gen = torch.Generator(device=dev).manual_seed(17)
+        kvs = []
+        for _ in range(2):
+            km = torch.randn((1, Nm, Hm, Dm), device=dev, generator=gen).to(torch.bfloat16)
+            vm = torch.randn((1, Nm, Hm, Dm), device=dev, generator=gen).to(torch.bfloat16)
+            kvs.append((km, vm, dreams.KVCache(km, vm, None)))
+        qx = torch.randn((1, Tq, Hm, Dm), device=dev, generator=gen).to(torch.bfloat16)
+        qp = torch.randn((1, Nm, Hm, Dm), device=dev, generator=gen).to(torch.bfloat16)
+        one = lambda n: torch.tensor([n], dtype=torch.int32, device=dev)
+        ox, op = torch.empty_like(qx), torch.empty_like(qp)
+        ent = torch.empty((1, Nm, Hm), dtype=torch.float32, device=dev)
+        ws_x = torch.zeros(max(16, dreams._lib().dreams_attention_workspace_size(
+            ctypes.byref(kvs[0][2]._c), 1, Tq, Hm, dreams.ATTN_FULL, 0)), dtype=torch.uint8, device=dev)
+        ws_p = torch.zeros(max(16, dreams._lib().dreams_attention_workspace_size(
+            ctypes.byref(kvs[0][2]._c), 1, Nm, Hm, dreams.ATTN_CAUSAL, 1)), dtype=torch.uint8, device=dev)
+        qlx, kvx, qlp, kvp = one(Tq), one(Nm), one(Nm), one(0)
+
+        def cross(i):
+            dreams.attention(qx, kvs[i % 2][2], qlx, kvx, Dm ** -0.5, dreams.ATTN_FULL, out=ox, workspace=ws_x,
+                             status=status)
+
+        def prefill(i):
+            o, _, e = dreams.attention(qp, kvs[i % 2][2], qlp, kvp, Dm ** -0.5, dreams.ATTN_CAUSAL, out=op,
+                                       want_entropy=True, workspace=ws_p, status=status)
+            return e
+
+        def time_it(fn, n):
+            for i in range(3):
+                fn(i)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            barrier()
+            e0.record(stream)
+            for i in range(n):
+                fn(i)
+            e1.record(stream)
+            barrier()
+            return e0.elapsed_time(e1) / n * 1000.0
+
+        x_us = time_it(cross, max(3, min(K, 50)))
+        p_us = time_it(prefill, max(3, min(K, 20)))
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item()):#x} (attention modes)")
+        ae = float(prefill(0).mean().item())
+        kv_bytes = 2 * Nm * Hm * Dm * 2
+        p_flops = 4.0 * Hm * Dm * Nm * (Nm + 1) / 2
+        bf16_burst, bf16_sust = bf16_peaks()
+        modes = {
+            "cross_attention": {"us": round(x_us, 1), "shape": "60 draft positions x 3392 target features, 32 heads",
+                                "bytes": kv_bytes, "GBps": round(kv_bytes / (x_us * 1e-6) / 1e9, 1)},
+            "prefill_entropy": {"us": round(p_us, 1), "shape": "causal 3392 tokens, 32 heads, entropy per row",
+                                "tflops": round(p_flops / (p_us * 1e-6) / 1e12, 1), "bound": "tensor",
+                                "frac_of_burst": round(p_flops / (p_us * 1e-6) / 1e12 / bf16_burst, 4),
+                                "AE_nats": round(ae, 4)},
+        }
+        del kvs, qx, qp
+
     ab, gb = attn_bytes(w), argmax_bytes(w)
     attn_avg_ms = sum(attn_ms) / K
     tail_avg_ms = sum(tail_ms) / K
@@ -454,6 +521,9 @@ def run_dreams(args, rank, world, local):
     if importance is not None:
         importance["frac_measured_hbm"] = round(importance["GBps"] / peak, 4)
         kernels["visual_importance"] = importance
+    if modes is not None:
+        modes["cross_attention"]["frac_measured_hbm"] = round(modes["cross_attention"]["GBps"] / peak, 4)
+        kernels.update(modes)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
