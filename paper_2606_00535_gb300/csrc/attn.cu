@@ -11,10 +11,11 @@
 // row block rb), one CTA per SM. A row block holds TB = 128 / G tree nodes
 // times the G query heads of the group, row = (t - rb*TB) * G + (h - gG), so
 // one pass over a K/V tile serves every query head of the GQA group and every
-// tree node of the block. With more than one sequence, a one-CTA kernel first
-// orders the (sequence, split) pairs longest first, so that the hardware,
-// which hands out CTAs in index order as SMs free up, schedules the items
-// longest-processing-time first.
+// tree node of the block. With more than one sequence the CTAs take the
+// (sequence, split) pairs longest first, so that the hardware, which hands out
+// CTAs in index order as SMs free up, schedules the items longest-processing-
+// time first: with up to 64 pairs each CTA ranks the pairs itself, with more a
+// one-CTA kernel orders them first.
 //
 // Roles (320 threads):
 //   warp 8, one thread  TMA producer: the Q block first (one 5-D box per
@@ -78,6 +79,7 @@ constexpr float RESCALE = 8.f; // log2 headroom of the reference maximum
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int MAX_SPLITS = 32; // KV splits per sequence (one merge lane each)
 constexpr int ORDER_THREADS = 1024;
+constexpr int RANK_PAIRS = 64;     // up to this many (sequence, split) pairs each CTA ranks them itself
 constexpr int ORDER_KEYS = 4096;  // item sizes (tiles) above this share the top bucket
 constexpr int PAST_TABLE = INT_MIN;  // page-table slot past the table: reads as zeros
 
@@ -100,7 +102,8 @@ struct AttnParams {
   float scale_log2;
   float *ws_o;     // [B][Hkv][nrb][nsplit][ROWS][D] unnormalised partial O
   float2 *ws_ml;   // [B][Hkv][nrb][nsplit][ROWS] (max in log2 units, sum)
-  int32_t *order;  // [B * nsplit] pair index b * nsplit + split, longest first; nullptr: natural order
+  int32_t *order;  // [B * nsplit] pair index b * nsplit + split, longest first; nullptr: see rank
+  int32_t rank;    // with no order: 1 = each CTA ranks the pairs itself (B * nsplit <= RANK_PAIRS), 0 = natural order
   int32_t *status;
   int32_t mode;    // ATTN_TREE, ATTN_FULL or ATTN_CAUSAL: which slots a query row attends
   float *ent;      // [B, T_max, Hq] attention entropy of each query row (nats), with the entropy kernels
@@ -238,6 +241,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   __shared__ int s_abort, s_zero, s_flag;
   __shared__ unsigned long long s_anc[64];
   __shared__ int s_jump[64];
+  __shared__ int s_key[RANK_PAIRS];
+  __shared__ int s_pair;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int per_pair = p.Hkv * p.nrb;
@@ -251,8 +256,46 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     // the order comes from the preceding kernel (programmatic dependent launch)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     pair = __ldcg(p.order + pair_pos);
+  } else if (p.rank) {
+    // few pairs: the CTA takes the pair of rank pair_pos in the order by KV
+    // tiles, largest first, ties by pair index (every CTA computes the same
+    // order, one pair per thread)
+    const int np = p.B * p.nsplit;
+    int key = 0;
+    if (tid < np) {
+      key = split_tiles(p, tid / p.nsplit, tid % p.nsplit);
+      s_key[tid] = key;
+    }
+    __syncthreads();
+    if (tid < np) {
+      int r = 0;
+      for (int f = 0; f < np; ++f) {
+        const int kf = s_key[f];
+        r += (kf > key) || (kf == key && f < tid);
+      }
+      if (r == pair_pos) s_pair = tid;
+    }
+    __syncthreads();
+    pair = s_pair;
   }
   const int b = pair / p.nsplit, split = pair - b * p.nsplit;
+  // The loads the prologue depends on go out together: the tree row (MMA
+  // warp) and the first page-table entries (producer), next to the lengths.
+  int par_pre[2] = {-1, -1};
+  if (warp == MMA_WARP && p.mode == ATTN_TREE) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int i = lane + 32 * h;
+      if (i < p.T_max) par_pre[h] = __ldg(p.parent + int64_t(b) * p.T_max + i);
+    }
+  }
+  int pn_pre[2] = {PAST_TABLE, PAST_TABLE};
+  if (tid == TMA_WARP * 32 && P.paged) {
+    const int pi = (split * p.chunk) >> 6;
+    const int32_t *prow = p.page_table + int64_t(b) * p.pages_per_seq;
+    if (pi < p.pages_per_seq) pn_pre[0] = __ldg(prow + pi);
+    if (pi + 1 < p.pages_per_seq) pn_pre[1] = __ldg(prow + pi + 1);
+  }
   const bool reporter = (rb == 0 && split == 0 && g == 0);
   const int T = __ldg(p.tree_len + b);
   const int L = __ldg(p.kv_len + b);
@@ -339,7 +382,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int i = lane + 32 * h;
-      par[h] = (i < T) ? __ldg(p.parent + int64_t(b) * p.T_max + i) : -1;
+      par[h] = (i < T) ? par_pre[h] : -1;
       if (i == 0) bad |= (par[h] != -1);
       else if (i < T) bad |= (par[h] < 0 || par[h] >= i);
     }
@@ -419,8 +462,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         return e;
       };
       int ring[CRD][2];
-      int pn0 = 0, pn1 = 0;
-      fetch(0, pn0, pn1);
+      int pn0 = pn_pre[0], pn1 = pn_pre[1];  // tile 0 (loaded at the start)
       int nk = 0, nv = 0;  // tiles issued into each ring
       uint32_t idle = 0;
       uint64_t t_idle = 0;
@@ -485,14 +527,12 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const uint64_t qd0 = tc::smem_desc_sw128(q_s, 16, 1024);
       const uint64_t kd0 = tc::smem_desc_sw128(k_s(0), 16, 1024);
       const uint64_t vd0 = tc::smem_desc_sw128(v_s(0), KV_REGION, 1024);
+      // The tensor pipe holds only a few MMAs, so the issuing thread must not
+      // stall between them: per tile it takes all its waits at once, then
+      // issues PV_j and QK_{j+2} (16 MMAs) back to back under one commit.
       // S_j = Q K_j^T into warpgroup (j % 2)'s S buffer
       auto qk = [&](int j) {
         const int ks = j % NK;
-        if (!tc::mbar_wait(kf0 + 8 * ks, (j / NK) & 1, abort_flag)) {
-          give_up();
-          return false;
-        }
-        tc::fence_after_sync();
         const uint32_t scol = 256u * (j & 1);
 #pragma unroll
         for (int k = 0; k < D / 16; ++k) {
@@ -501,32 +541,49 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           const uint64_t bd = kd0 + ((uint32_t(ks) * KV_TILE + (k >> 2) * KV_REGION + off) >> 4);
           tc::mma_ss(tmem + scol, ad, bd, IDESC_QK, k > 0 ? 1u : 0u);
         }
-        tc::mma_commit(bs0 + 8 * (j & 1));
-        tc::mma_commit(ke0 + 8 * ks);
-        return true;
       };
-      // O_w += P_j V_j once warpgroup w = j % 2 has written P_j
+      // O_w += P_j V_j, w = j % 2
       auto pv = [&](int j) {
         const int w = j & 1, ii = j >> 1, vs = j % NV;
-        if (!tc::mbar_wait(bp0 + 8 * w, ii & 1, abort_flag) || !tc::mbar_wait(vf0 + 8 * vs, (j / NV) & 1, abort_flag)) {
-          give_up();
-          return false;
-        }
-        tc::fence_after_sync();
         const uint32_t scol = 256u * w, ocol = 256u * w + 128u;
 #pragma unroll
         for (int ks = 0; ks < KT / 16; ++ks) {
           const uint64_t bd = vd0 + ((uint32_t(vs) * KV_TILE + ks * 2048) >> 4);
           tc::mma_ts(tmem + ocol, tmem + scol + ks * 8, bd, IDESC_PV, (ii > 0 || ks > 0) ? 1u : 0u);
         }
-        tc::mma_commit(ve0 + 8 * vs);
-        return true;
       };
-      bool ok = tc::mbar_wait(bq, 0, abort_flag);
+      auto kwait = [&](int j) { return tc::mbar_wait(kf0 + 8 * (j % NK), (j / NK) & 1, abort_flag); };
+      bool ok = tc::mbar_wait(bq, 0, abort_flag) && kwait(0);
+      if (ok) {
+        tc::fence_after_sync();
+        qk(0);
+        tc::mma_commit(bs0);
+      }
+      if (ok && ntiles > 1) {
+        ok = kwait(1);
+        if (ok) {
+          tc::fence_after_sync();
+          qk(1);
+          tc::mma_commit(bs0 + 8);
+        }
+      }
+      // The commit after QK_{j+2} also covers PV_j (the pipe completes in
+      // order): the softmax warps, woken by it, release the stages of K_{j+2}
+      // and V_j to the producer.
+      for (int j = 0; j < ntiles && ok; ++j) {
+        const int w = j & 1;
+        // the copies have usually landed; P_j, the one to wait for, comes last
+        ok = (j + 2 >= ntiles || kwait(j + 2)) && tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag) &&
+             tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag);
+        if (!ok) break;
+        tc::fence_after_sync();
+        pv(j);
+        if (j + 2 < ntiles) {
+          qk(j + 2);
+          tc::mma_commit(bs0 + 8 * w);
+        }
+      }
       if (!ok) give_up();
-      // QK of tile j + 2 reuses the S buffer of tile j, so it follows PV_j
-      ok = ok && qk(0) && (ntiles < 2 || qk(1));
-      for (int j = 0; j < ntiles && ok; ++j) ok = pv(j) && (j + 2 >= ntiles || qk(j + 2));
       tc::mma_commit(bdrain);
       tc::mbar_wait(bdrain, 0, &s_zero);
     }
@@ -547,8 +604,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         break;
       }
       // S_j is complete, and so (issued earlier) is this warpgroup's previous
-      // PV, so O may be rescaled below
+      // PV, so O may be rescaled below. The K stage of tile j and the V stage
+      // of tile j - 2 (read by that PV) go back to the producer.
       tc::fence_after_sync();
+      if (warp == 4 * wg && lane == 0) {
+        tc::mbar_arrive(ke0 + 8 * (j % NK));
+        if (j >= 2) tc::mbar_arrive(ve0 + 8 * ((j - 2) % NV));
+      }
       uint32_t sv[KT];
 #pragma unroll
       for (int q4 = 0; q4 < KT / 32; ++q4)
@@ -899,7 +961,8 @@ struct AttnPlan {
   int nrb;
   int nsplit;
   int chunk;
-  bool ordered;
+  bool ordered;  // a separate kernel orders the pairs
+  bool ranked;   // each CTA ranks the pairs itself
   size_t ws_o_bytes, ws_ml_bytes, ws_w_bytes, order_bytes;
   size_t ws_bytes;
 };
@@ -942,7 +1005,8 @@ AttnPlan plan(const dreams_kv_cache_t *kv, int B, int T_max, int Hq, bool ent) {
     pl.ws_ml_bytes = align_up(slots * sizeof(float2), 256);
     if (ent) pl.ws_w_bytes = align_up(slots * sizeof(float), 256);
   }
-  pl.ordered = B > 1;
+  pl.ranked = B > 1 && int64_t(B) * pl.nsplit <= RANK_PAIRS;
+  pl.ordered = B > 1 && !pl.ranked;
   if (pl.ordered) pl.order_bytes = align_up(size_t(B) * pl.nsplit * sizeof(int32_t), 256);
   pl.ws_bytes = pl.ws_o_bytes + pl.ws_ml_bytes + pl.ws_w_bytes + pl.order_bytes;
   return pl;
@@ -1135,6 +1199,7 @@ dreams_status_t attention_impl(const void *q, const dreams_kv_cache_t *kv, int32
     if (want_ent) p.ws_w = reinterpret_cast<float *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes);
   }
   if (pl.ordered) p.order = reinterpret_cast<int32_t *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes + pl.ws_w_bytes);
+  p.rank = pl.ranked ? 1 : 0;
   p.status = status_word;
   const void *k = static_cast<const __nv_bfloat16 *>(kv->k) + int64_t(layer) * kv->layer_stride;
   const void *v = static_cast<const __nv_bfloat16 *>(kv->v) + int64_t(layer) * kv->layer_stride;

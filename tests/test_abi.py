@@ -52,8 +52,11 @@ def test_workspace_sizes(lib):
     n = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 32)
     assert n > 0 and n % 256 == 0
     tr = dreams._Tree(16, 16, 16, 16, 16, 64)
-    # several sequences: the longest-first order of the work items needs room too
-    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32) >= 16 * 4
+    # 16 sequences, one split each: the CTAs rank the 16 pairs themselves, no workspace
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32) == 0
+    # 128 sequences: the longest-first order of the work items needs room
+    tr = dreams._Tree(16, 16, 16, 16, 128, 64)
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(tr), 32) >= 128 * 4
     bad = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
     assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(bad), ctypes.byref(tr), 30) == 0
     assert lib.dreams_vocab_argmax_workspace_size(768, 128256) >= 0
@@ -61,9 +64,9 @@ def test_workspace_sizes(lib):
 
 
 def test_attention_workspace_covers_every_row_block(lib):
-    """A CTA takes a pair of row blocks, but the split partials are kept per
-    row block: with 5 query heads per KV head and 64 nodes there are 3 row
-    blocks (25 nodes each), so one split needs 3 x 128 rows of (O, m, l)."""
+    """The split partials are kept per row block: with 5 query heads per KV
+    head and 64 nodes there are 3 row blocks (25 nodes each), so one split
+    needs 3 x 128 rows of (O, m, l)."""
     kvc = dreams._KVCache(16, 16, 1, 0, 1, 128, 2304, None, 0, 0, 0)
     one = dreams._Tree(16, 16, 16, 16, 1, 64)
     ws = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 5)
@@ -73,14 +76,20 @@ def test_attention_workspace_covers_every_row_block(lib):
 
 def test_attention_launch_count(lib):
     """One sequence: the attention, plus a merge when the KV range is split
-    (the workspace then holds the partials); several sequences add the
-    longest-first ordering pass; rejected shapes make no launch."""
+    (the workspace then holds the partials). Several sequences are taken
+    longest first: up to 64 (sequence, split) pairs each CTA ranks them
+    itself, beyond that a separate ordering pass runs first (its order lives
+    in the workspace). Rejected shapes make no launch."""
     kvc = dreams._KVCache(16, 16, 1, 0, 8, 128, 6080, None, 0, 0, 0)
     one = dreams._Tree(16, 16, 16, 16, 1, 64)
     split = lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(one), 32) > 0
     assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(one), 32) == 1 + int(split)
-    many = dreams._Tree(16, 16, 16, 16, 16, 64)
-    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(many), 32) >= 2
+    many = dreams._Tree(16, 16, 16, 16, 16, 64)  # 16 sequences x 8 KV heads x 2 row blocks: one split
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(many), 32) == 0
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(many), 32) == 1
+    lots = dreams._Tree(16, 16, 16, 16, 128, 64)  # 128 pairs: the ordering pass
+    assert lib.dreams_tree_verify_attn_workspace_size(ctypes.byref(kvc), ctypes.byref(lots), 32) >= 128 * 4
+    assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(lots), 32) == 2
     assert lib.dreams_tree_verify_attn_launches(ctypes.byref(kvc), ctypes.byref(many), 30) == 0
     d96 = dreams._KVCache(16, 16, 1, 0, 8, 96, 6080, None, 0, 0, 0)
     assert lib.dreams_tree_verify_attn_launches(ctypes.byref(d96), ctypes.byref(many), 32) == 0

@@ -76,10 +76,10 @@ def test_attention_mask_sensitive(dreams, name, L, key_scale):
     (2, 14, 2, 128, 40, 300, 400),    # group of 7 heads: 18 nodes (126 rows) per row block
     (1, 100, 1, 64, 5, 100, 200),     # group of 100 heads: one node per row block
     (2, 128, 1, 64, 3, 50, 100),      # the largest group (128 heads)
-    (1, 3, 1, 128, 64, 2000, 2304),   # 2 row blocks in one CTA, KV range split
-    (1, 5, 1, 128, 64, 2000, 2304),   # 3 row blocks: a pair and a lone block, KV range split
-    (1, 6, 1, 128, 64, 2000, 2304),   # 4 row blocks: two pairs, KV range split
-    (2, 10, 2, 64, 61, 1500, 1600),   # head dim 64, pairs, ragged split tail
+    (1, 3, 1, 128, 64, 2000, 2304),   # 2 row blocks, KV range split
+    (1, 5, 1, 128, 64, 2000, 2304),   # 3 row blocks, KV range split
+    (1, 6, 1, 128, 64, 2000, 2304),   # 4 row blocks, KV range split
+    (2, 10, 2, 64, 61, 1500, 1600),   # head dim 64, ragged split tail
 ])
 def test_attention_edge_shapes(dreams, B, Hq, Hkv, D, T, L, cap):
     rng = np.random.default_rng(B * 1000 + T)
@@ -127,6 +127,34 @@ def test_attention_uneven_lengths(dreams):
     kv = dreams.KVCache(k.cuda(), v.cuda())
     tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
                        torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    st = _status()
+    out, lse = dreams.tree_verify_attn(q.cuda(), kv, tree, scale, want_lse=True, status=st)
+    ref, ref_lse, sel, ost = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v), oracle.KVLayout(cap, Hkv, D),
+                                                   par, tl, kl, Hq, scale)
+    assert ost == 0 and int(st.item()) == 0
+    compare_attention(out, lse, ref, ref_lse, sel)
+
+
+@pytest.mark.parametrize("B", [64, 80])
+def test_attention_many_sequences(dreams, B):
+    """64 (sequence, split) pairs are the most each CTA ranks itself; 80 take
+    the separate ordering pass. Lengths repeat, so equal work sizes tie."""
+    rng = np.random.default_rng(B)
+    Hq, Hkv, D, T, cap = 4, 2, 64, 8, 320
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    tl = rng.integers(1, T + 1, B).astype(np.int32)
+    for b in range(B):
+        par[b, tl[b]:] = -1
+    kl = rng.choice([0, 5, 127, 128, 200, 311], B).astype(np.int32)
+    kl = np.minimum(kl, cap - tl)
+    q = W.bf16(rng.standard_normal((B, T, Hq, D), dtype=np.float32))
+    k = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    v = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    scale = 1.0 / np.sqrt(D)
+    kv = dreams.KVCache(k.cuda(), v.cuda())
+    tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
+                       torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    assert dreams.tree_verify_attn_launches(kv, tree, Hq) == (1 if B <= 64 else 2)
     st = _status()
     out, lse = dreams.tree_verify_attn(q.cuda(), kv, tree, scale, want_lse=True, status=st)
     ref, ref_lse, sel, ost = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v), oracle.KVLayout(cap, Hkv, D),
