@@ -527,9 +527,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const uint64_t qd0 = tc::smem_desc_sw128(q_s, 16, 1024);
       const uint64_t kd0 = tc::smem_desc_sw128(k_s(0), 16, 1024);
       const uint64_t vd0 = tc::smem_desc_sw128(v_s(0), KV_REGION, 1024);
-      // The tensor pipe holds only a few MMAs, so the issuing thread must not
-      // stall between them: per tile it takes all its waits at once, then
-      // issues PV_j and QK_{j+2} (16 MMAs) back to back under one commit.
+      // The tensor pipe queues only about one MMA, so any latency in the
+      // issuing thread between MMAs idles it: per tile the thread takes one
+      // wait, then issues PV_j and QK_{j+2} (16 MMAs) under one commit.
       // S_j = Q K_j^T into warpgroup (j % 2)'s S buffer
       auto qk = [&](int j) {
         const int ks = j % NK;
@@ -572,9 +572,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       // and V_j to the producer.
       for (int j = 0; j < ntiles && ok; ++j) {
         const int w = j & 1;
-        // the copies have usually landed; P_j, the one to wait for, comes last
-        ok = (j + 2 >= ntiles || kwait(j + 2)) && tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag) &&
-             tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag);
+        // P_j: the softmax warps arrive once one of them has also seen V_j
+        // and K_{j+2} land
+        ok = tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag);
         if (!ok) break;
         tc::fence_after_sync();
         pv(j);
@@ -723,6 +723,18 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
           tc::tmem_st32(tl + 128 + c4 * 32, ov);
         }
+      }
+      // One thread also waits for the copies the MMA thread needs next, V_j
+      // and K_{j+2} (usually landed by now; the wait overlaps the TMEM
+      // stores): the MMA thread then waits for P_j alone.
+      bool kv_ok = true;
+      if (warp == 4 * wg && lane == 0)
+        kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag) &&
+                (j + 2 >= ntiles || tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag));
+      if (!__all_sync(0xffffffffu, kv_ok)) {
+        give_up();
+        ok = false;
+        break;
       }
       tc::tmem_wait_st();
       tc::fence_before_sync();
