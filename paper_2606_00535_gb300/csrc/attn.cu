@@ -25,15 +25,15 @@
 //                       swizzle). It polls both rings without blocking and
 //                       keeps V a tile behind K (QK^T of tile j + 1 runs
 //                       before PV of tile j); page-table entries are loaded
-//                       one tile ahead. A K stage is released as soon as its QK^T
-//                       has run, a V stage after its PV.
+//                       one tile ahead.
 //   warp 9, one thread  MMA issuer: S = Q K^T (M128 N128, K-major operands) into
 //                       TMEM, O += P V (M128 N=D, P read from TMEM, V as an
 //                       MN-major operand). Tile j goes to warpgroup j % 2, and
 //                       the QK^T of tile j + 2 follows the PV of tile j (they
-//                       share that warpgroup's S/P columns). A tcgen05.mma
-//                       costs at least ~50 ns, so 128-token tiles halve the
-//                       QK^T instructions of 64-token ones.
+//                       share that warpgroup's S/P columns). The tensor pipe
+//                       queues about one MMA, so the thread must not stall
+//                       between MMAs: per tile it waits once (for P_j), then
+//                       issues PV_j and QK_{j+2} (16 MMAs) under one commit.
 //   warps 0-3, 4-7      two softmax warpgroups, one query row per thread. A
 //                       warpgroup owns one S/P buffer and its own O in TMEM
 //                       (256 columns each), so the two alternate over the
@@ -42,8 +42,13 @@
 //                       exponentiates with ex2.approx against a reference
 //                       maximum that is raised only when a tile's maximum
 //                       exceeds it by 2^8 (and only then rescales its O), and
-//                       writes P as bf16 over S. Warps whose rows are all
-//                       padding sit out.
+//                       writes P as bf16 over S. Woken by the commit after
+//                       QK_j (which also covers PV_{j-2}), one thread
+//                       releases the K stage of tile j and the V stage of
+//                       tile j - 2 to the producer; before the warpgroup
+//                       signals P_j it waits for V_j and K_{j+2} to land, so
+//                       that the MMA thread needs no other wait. Warps whose
+//                       rows are all padding sit out.
 // At the end the two warpgroups combine their (m, l, O) by log-sum-exp into a
 // swizzled staging copy in the idle shared-memory rings, and all 256 threads
 // write it out in row order (16-byte coalesced stores): the output, or the
