@@ -62,6 +62,10 @@ def parse():
                     help="untimed steps run while the clock sampler starts (0 under a profiler)")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every call from Python in the timed loop instead of replaying CUDA graphs")
+    ap.add_argument("--flush-l2", action="store_true",
+                    help="before every timed step (outside its events) write a buffer twice the size of L2, then "
+                         "read another as large, so that L2 holds only clean unrelated lines; average the per-step "
+                         "times: for workloads whose inputs fit in L2")
     return ap.parse_args()
 
 
@@ -281,9 +285,16 @@ def run_dreams(args, rank, world, local):
 
     K = args.steps
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev) if args.flush_l2 else None
+    flush_read = torch.zeros(L2_BYTES // 2, dtype=torch.float32, device=dev) if args.flush_l2 else None
     barrier()
     t0 = time.time()
     for i in range(K):
+        if flush_buf is not None:
+            # the write evicts the step's inputs; the read then evicts the
+            # dirty lines, so the step pays no write-back of the flush
+            flush_buf.fill_(i & 255)
+            flush_read.sum()
         step(i % 2, evs[i])
     barrier()
     wall = time.time() - t0
@@ -292,7 +303,9 @@ def run_dreams(args, rank, world, local):
     total_ms = evs[0][0].elapsed_time(evs[-1][2])
     attn_ms = [e[0].elapsed_time(e[1]) for e in evs]
     tail_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    ms_per_step = total_ms / K
+    # back to back: the whole timed span over K; with the flushes between
+    # steps: the mean of the steps' own spans
+    ms_per_step = total_ms / K if flush_buf is None else sum(e[0].elapsed_time(e[2]) for e in evs) / K
     if world > 1:
         import torch.distributed as dist
         t = torch.tensor([ms_per_step], device=dev)
@@ -539,7 +552,11 @@ def run_dreams(args, rank, world, local):
             "config": {"workload": w.spec.description, "name": w.spec.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv,
                        "D": w.D, "T_max": w.T_max, "V": w.V, "logits": w.logits_dtype,
                        "kv_tokens": int((w.kv_len + w.tree_len).sum()), "tree_nodes": int(w.tree_len.sum()),
-                       "l2": f"inputs larger than L2: 2 rotating copies of {copy_bytes / 2**20:.0f} MiB each",
+                       "l2": (f"L2 flushed before every step ({2 * L2_BYTES / 2**20:.0f} MiB written, then as "
+                              f"much read, outside the step's events); 2 rotating input copies of "
+                              f"{copy_bytes / 2**20:.0f} MiB each"
+                              if args.flush_l2 else
+                              f"inputs larger than L2: 2 rotating copies of {copy_bytes / 2**20:.0f} MiB each"),
                        "parallelism": f"replicas x{world}", "launch": launch_mode},
             "e2e": e2e, "gpu_launches": launches_per_step * K, "roofline": roofline, "kernels": kernels,
             "tau_mean_accept_len": None, "clocks": clk, "cpu_baseline": cpu, "wall_s": round(wall, 3),
