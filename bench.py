@@ -174,6 +174,24 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# ---------------------------------------------------------------- replicas
+def rank_seed(name: str, rank: int):
+    """Seed of a rank's inputs: rank 0 draws the workload's own seeded inputs,
+    every other rank a seed of its own (replicas verify different batches)."""
+    return None if rank == 0 else 20260 + 97 * rank + W.SPEC_BY_NAME[name].index
+
+
+def max_over_ranks(x: float, device) -> float:
+    """The largest x over the ranks of the default process group (x itself
+    without one): the job's step time is its slowest replica's."""
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ---------------------------------------------------------------- dreams arm
 def run_dreams(args, rank, world, local):
     import paper_2606_00535_gb300 as dreams
@@ -183,7 +201,7 @@ def run_dreams(args, rank, world, local):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
 
-    w = W.make(args.config, seed=None if rank == 0 else 20260 + 97 * rank + W.SPEC_BY_NAME[args.config].index)
+    w = W.make(args.config, seed=rank_seed(args.config, rank))
     max_path = w.max_path
     copies = []
     for _ in range(2):
@@ -306,11 +324,7 @@ def run_dreams(args, rank, world, local):
     # back to back: the whole timed span over K; with the flushes between
     # steps: the mean of the steps' own spans
     ms_per_step = total_ms / K if flush_buf is None else sum(e[0].elapsed_time(e[2]) for e in evs) / K
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms_per_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_per_step = float(t.item())
+    ms_per_step = max_over_ranks(ms_per_step, dev)
 
     # ---- e2e through the public API with host buffers
     e2e = None
