@@ -34,6 +34,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA, ERR_SCRATCH_LIMIT
 NOALLOC_ARGMAX_MAX_ROWS = 16384
 F32, BF16 = 0, 1
 DATA_BAD_PARENT, DATA_BAD_TREE_LEN, DATA_BAD_KV_LEN, DATA_BAD_PAGE, DATA_BAD_PATH = 1, 2, 4, 8, 16
+DATA_TIMEOUT = 0x20  # a kernel gave up waiting on its own pipeline
 
 
 class DreamsError(RuntimeError):

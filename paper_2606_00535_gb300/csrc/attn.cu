@@ -123,6 +123,14 @@ constexpr int ATTN_CAUSAL = 2;  // slots 0 .. kv_len + t for query t (prefill se
 // causal), or the prefix alone (full).
 __device__ __forceinline__ int key_total(const AttnParams &p, int L, int T) { return p.mode == ATTN_FULL ? L : L + T; }
 
+// A read-only global load issued where it stands (the compiler may not sink it
+// to the value's first use).
+__device__ __forceinline__ int ld_issue_now(const int32_t *ptr) {
+  int v;
+  asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(ptr));
+  return v;
+}
+
 struct TcParams {
   CUtensorMap tmap_q;
   CUtensorMap tmap_k;
@@ -284,14 +292,16 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     pair = s_pair;
   }
   const int b = pair / p.nsplit, split = pair - b * p.nsplit;
-  // The loads the prologue depends on go out together: the tree row (MMA
-  // warp) and the first page-table entries (producer), next to the lengths.
+  // The loads the prologue depends on go out together: the tree row (softmax
+  // warp 0, which builds the masks) and the first page-table entries
+  // (producer), next to the lengths. Volatile, so that they are issued here
+  // and not where their values are first used.
   int par_pre[2] = {-1, -1};
-  if (warp == MMA_WARP && p.mode == ATTN_TREE) {
+  if (warp == 0 && p.mode == ATTN_TREE) {
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int i = lane + 32 * h;
-      if (i < p.T_max) par_pre[h] = __ldg(p.parent + int64_t(b) * p.T_max + i);
+      if (i < p.T_max) par_pre[h] = ld_issue_now(p.parent + int64_t(b) * p.T_max + i);
     }
   }
   int pn_pre[2] = {PAST_TABLE, PAST_TABLE};
@@ -349,6 +359,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     tc::mbar_init(bdrain, 1);
     s_abort = 0;
     s_zero = 0;
+    s_flag = 0;
     tc::fence_barrier_init();
   }
   if (warp == MMA_WARP) {
@@ -372,17 +383,16 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     }
   };
 
-  // While the producer streams Q, K and V, the MMA warp checks the tree and
-  // builds the ancestor masks; named barrier 2 (MMA warp + softmax warps)
-  // publishes them.
+  // While the producer streams Q, K and V and the MMA thread starts on them,
+  // softmax warp 0 checks the tree and builds the ancestor masks; named
+  // barrier 2 (the softmax warps) publishes them before the first tile. A
+  // malformed tree stops the producer and the MMA thread through the abort
+  // flag.
   const int wg = warp >> 2;                  // softmax warpgroup (warps 0-7)
   const int row = 32 * (warp & 3) + lane;    // TMEM lane = query row
   const bool real_row = row < rows_blk;
   const int t_row = t0 + row / p.G;
-  if (warp == MMA_WARP && p.mode != ATTN_TREE) {
-    if (lane == 0) s_flag = 0;  // no tree: every key set is a prefix of the slots
-    named_sync(2, 288);
-  } else if (warp == MMA_WARP) {
+  if (warp == 0 && p.mode == ATTN_TREE) {
     int par[2], bad = 0;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -426,11 +436,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         __syncwarp();
       }
     }
-    named_sync(2, 288);
-  } else if (warp < 8) {
-    named_sync(2, 288);
   }
-  const bool tree_ok = (warp == TMA_WARP) || !s_flag;
+  if (warp < 8) named_sync(2, 256);
+  // the producer and the MMA thread learn of a malformed tree from the abort flag
+  const bool tree_ok = warp >= 8 || !s_flag;
 
   float m_ref = -INFINITY, l = 0.f;  // this thread's row state (softmax warps)
   float wsum = 0.f;                  // entropy: sum_j P_j (x_j - m_ref), x = scaled score in log2 units

@@ -163,6 +163,43 @@ def test_attention_many_sequences(dreams, B):
     compare_attention(out, lse, ref, ref_lse, sel)
 
 
+@pytest.mark.parametrize("B", [1, 3])
+def test_attention_malformed_tree(dreams, B):
+    """A sequence whose parent array is malformed (a parent after its child)
+    is flagged and its output rows are left untouched, while the MMAs and
+    copies of its CTAs stop through the abort flag; the other sequences are
+    computed as usual. B = 1 splits the KV range, B = 3 ranks the pairs."""
+    rng = np.random.default_rng(90 + B)
+    Hq, Hkv, D, T, cap = 8, 2, 128, 40, 1536
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    bad = B // 2
+    good_par = par.copy()
+    par[bad, 7] = 9
+    tl = np.full(B, T, np.int32)
+    kl = np.array([1000, 700, 1200][:B], np.int32)
+    q = W.bf16(rng.standard_normal((B, T, Hq, D), dtype=np.float32))
+    k = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    v = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    scale = 1.0 / np.sqrt(D)
+    kv = dreams.KVCache(k.cuda(), v.cuda())
+    tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
+                       torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    out = torch.full((B, T, Hq, D), 7.0, dtype=torch.bfloat16, device="cuda")
+    st = _status()
+    out, lse = dreams.tree_verify_attn(q.cuda(), kv, tree, scale, out=out, want_lse=True, status=st)
+    s = int(st.item())
+    assert s & dreams.DATA_BAD_PARENT and not s & dreams.DATA_TIMEOUT, hex(s)
+    assert (out[bad].float() == 7.0).all()
+    others = [b for b in range(B) if b != bad]
+    if others:
+        sel = np.array([(b, t, h) for b in others for t in range(T) for h in range(Hq)], np.int32)
+        ref, ref_lse, sel, ost = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v),
+                                                       oracle.KVLayout(cap, Hkv, D), good_par, tl, kl, Hq, scale,
+                                                       sel=sel)
+        assert ost == 0
+        compare_attention(out, lse, ref, ref_lse, sel)
+
+
 def test_attention_paged_equals_contiguous(dreams):
     """The batched workload copied into a contiguous cache gives bit-identical
     results to its paged form."""
