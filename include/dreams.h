@@ -137,8 +137,10 @@ typedef struct dreams_tree {
 size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
                                               int32_t Hq);
 /* Kernel launches one dreams_tree_verify_attn call with these shapes makes
- * (1 to 3: an ordering pass for B > 1, the attention, a merge of the KV
- * splits when the cache is split); 0 for shapes the call rejects. */
+ * (1 to 3: an ordering pass when more than 64 (sequence, KV split) pairs are
+ * scheduled longest first (up to 64, every CTA ranks them itself), the
+ * attention, a merge of the KV splits when the cache is split); 0 for shapes
+ * the call rejects. */
 int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int32_t Hq);
 dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
                                         const dreams_tree_t *tree, int32_t Hq, float scale, void *out,
