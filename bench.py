@@ -326,20 +326,40 @@ def run_dreams(args, rank, world, local):
     ms_per_step = total_ms / K if flush_buf is None else sum(e[0].elapsed_time(e[2]) for e in evs) / K
     ms_per_step = max_over_ranks(ms_per_step, dev)
 
-    # ---- e2e through the public API with host buffers
+    # ---- e2e through the public API with host buffers. The inputs of a step
+    # are the tree arrays and the q and logits rows of its real tree nodes
+    # (rows t >= tree_len[b] are padding): per sequence one contiguous slice
+    # of each. The logits travel on a second stream while the attention runs.
     e2e = None
     if not args.no_e2e:
         c = copies[0]
         host_in = {n: c[n].cpu().pin_memory() for n in ("q", "logits", "parent", "tokens", "tree_len", "kv_len")}
         host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (c["outs"][0], c["outs"][2],
                                                                              c["outs"][3])]
-        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        small = ("parent", "tokens", "tree_len", "kv_len")
+        tl_host = [int(x) for x in host_in["tree_len"]]
+        row_bytes = {n: host_in[n][0, 0].numel() * host_in[n].element_size() for n in ("q", "logits")}
+        h2d = (sum(host_in[n].numel() * host_in[n].element_size() for n in small)
+               + sum(tl_host) * (row_bytes["q"] + row_bytes["logits"]))
         d2h = sum(t.numel() * t.element_size() for t in host_out)
+        copy_stream = torch.cuda.Stream(dev)
+        # (device, pinned host) slice pairs, made once: the long logits copies
+        # are issued first, so that the copy engine is never left waiting on
+        # Python between them
+        rows_logits = [(c["logits"][b, :t], host_in["logits"][b, :t]) for b, t in enumerate(tl_host) if t > 0]
+        rows_q = [(c["q"][b, :t], host_in["q"][b, :t]) for b, t in enumerate(tl_host) if t > 0]
 
         def e2e_step():
-            for n, t in host_in.items():
-                c[n].copy_(t, non_blocking=True)
+            copy_stream.wait_stream(stream)  # the previous step has read its logits
+            with torch.cuda.stream(copy_stream):
+                for d, h in rows_logits:
+                    d.copy_(h, non_blocking=True)
+            for n in small:
+                c[n].copy_(host_in[n], non_blocking=True)
+            for d, h in rows_q:
+                d.copy_(h, non_blocking=True)
             attn_call(c)  # through the public API, launched from Python
+            stream.wait_stream(copy_stream)
             step_call(c)
             for h, d in zip(host_out, (c["outs"][0], c["outs"][2], c["outs"][3])):
                 h.copy_(d, non_blocking=True)
