@@ -628,53 +628,51 @@ struct WalkOut {
   int bad;  // data-error bits
 };
 
-// One warp. Reads the sequence's parent / tokens / predictions, writes the
-// accepted path into s_path[0..n]. Pred rows may have been written by other
-// CTAs of this grid, so they are read through L2.
-__device__ WalkOut tree_walk_warp(const int32_t *par_row, const int32_t *tok_row, const int32_t *pred_row, int T,
-                                  int max_path, int32_t *s_path) {
-  __shared__ int s_good[64], s_dist[64], s_jump[64];
+// The tree alone, one warp, two nodes per lane (i = lane, lane + 32): each
+// node's parent, draft token, depth and ancestor set (itself included), by
+// pointer jumping. Needs no prediction, so the verification tail computes it
+// before waiting for the argmax grid.
+struct TreeShape {
+  int par[2], tok[2], dist[2];
+  unsigned long long anc[2];
+  int bad;  // DREAMS_DATA_BAD_PARENT or 0
+};
+
+__device__ TreeShape tree_shape_warp(const int32_t *par_row, const int32_t *tok_row, int T) {
+  __shared__ int s_dist[64], s_jump[64];
   __shared__ unsigned long long s_anc[64];
   const int lane = threadIdx.x & 31;
-  int par[2], tok[2], pred[2], bad = 0;
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int i = lane + 32 * h;
-    par[h] = (i < T) ? __ldg(par_row + i) : -1;
-    tok[h] = (i < T) ? __ldg(tok_row + i) : 0;
-    pred[h] = (i < T) ? __ldcg(pred_row + i) : 0;
-    if (i == 0) bad |= (par[h] != -1);
-    else if (i < T) bad |= (par[h] < 0 || par[h] >= i);
-  }
-  if (__any_sync(0xffffffffu, bad)) return {-1, DREAMS_DATA_BAD_PARENT};
-  // pred of each node's parent, through shared memory
-  __shared__ int s_pred[64];
-  s_pred[lane] = pred[0];
-  s_pred[lane + 32] = pred[1];
-  __syncwarp();
-  int good[2], dist[2], jump[2];
-  unsigned long long anc[2];
+  TreeShape ts;
+  int bad = 0, jump[2];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int i = lane + 32 * h;
     const bool live = i < T;
-    good[h] = (i == 0) ? 1 : (live && tok[h] == s_pred[par[h]]);
-    dist[h] = (i == 0 || !live) ? 0 : 1;
-    jump[h] = live ? par[h] : -1;
-    anc[h] = 1ull << i;
-    s_good[i] = good[h];
-    s_dist[i] = dist[h];
+    ts.par[h] = live ? __ldg(par_row + i) : -1;
+    ts.tok[h] = live ? __ldg(tok_row + i) : 0;
+    if (i == 0) bad |= (ts.par[h] != -1);
+    else if (live) bad |= (ts.par[h] < 0 || ts.par[h] >= i);
+  }
+  ts.bad = __any_sync(0xffffffffu, bad) ? DREAMS_DATA_BAD_PARENT : 0;
+  if (ts.bad) return ts;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i = lane + 32 * h;
+    const bool live = i < T;
+    ts.dist[h] = (i == 0 || !live) ? 0 : 1;
+    jump[h] = live ? ts.par[h] : -1;
+    ts.anc[h] = 1ull << i;
+    s_dist[i] = ts.dist[h];
     s_jump[i] = jump[h];
-    s_anc[i] = anc[h];
+    s_anc[i] = ts.anc[h];
   }
   __syncwarp();
   for (int r = 0; r < 6; ++r) {
-    int gg[2], dd[2], jj[2];
+    int dd[2], jj[2];
     unsigned long long aa[2];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int j = jump[h];
-      gg[h] = j >= 0 ? s_good[j] : 1;
       dd[h] = j >= 0 ? s_dist[j] : 0;
       jj[h] = j >= 0 ? s_jump[j] : -1;
       aa[h] = j >= 0 ? s_anc[j] : 0ull;
@@ -683,22 +681,49 @@ __device__ WalkOut tree_walk_warp(const int32_t *par_row, const int32_t *tok_row
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int i = lane + 32 * h;
-      good[h] &= gg[h];
-      dist[h] += dd[h];
+      ts.dist[h] += dd[h];
       jump[h] = jj[h];
-      anc[h] |= aa[h];
-      s_good[i] = good[h];
-      s_dist[i] = dist[h];
+      ts.anc[h] |= aa[h];
+      s_dist[i] = ts.dist[h];
       s_jump[i] = jump[h];
-      s_anc[i] = anc[h];
+      s_anc[i] = ts.anc[h];
     }
     __syncwarp();
   }
+  return ts;
+}
+
+// The walk over a valid tree shape, one warp: a node matches when its draft
+// token equals its parent's prediction (the root always matches); a node is
+// accepted when every node of its root path matches. Writes the accepted
+// path into s_path[0..n]. Pred rows may have been written by other CTAs of
+// this grid or by the preceding grid, so they are read through L2.
+__device__ WalkOut tree_walk_finish(const TreeShape &ts, const int32_t *pred_row, int T, int max_path,
+                                    int32_t *s_path) {
+  __shared__ int s_pred[64];
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i = lane + 32 * h;
+    s_pred[i] = (i < T) ? __ldcg(pred_row + i) : 0;
+  }
+  __syncwarp();
+  bool match[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i = lane + 32 * h;
+    match[h] = (i == 0) || (i < T && ts.tok[h] == s_pred[ts.par[h]]);
+  }
+  const unsigned long long mm = uint64_t(__ballot_sync(0xffffffffu, match[0])) |
+                                (uint64_t(__ballot_sync(0xffffffffu, match[1])) << 32);
+  bool good[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) good[h] = lane + 32 * h < T && (ts.anc[h] & ~mm) == 0ull;
   // longest matching depth, cut to max_path - 1 drafts
   int n = 0;
 #pragma unroll
   for (int h = 0; h < 2; ++h)
-    if (lane + 32 * h < T && good[h]) n = max(n, dist[h]);
+    if (good[h]) n = max(n, ts.dist[h]);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) n = max(n, __shfl_xor_sync(0xffffffffu, n, off));
   n = min(n, max_path - 1);
@@ -706,20 +731,28 @@ __device__ WalkOut tree_walk_warp(const int32_t *par_row, const int32_t *tok_row
   unsigned long long mark = 0ull;
 #pragma unroll
   for (int h = 0; h < 2; ++h)
-    if (lane + 32 * h < T && good[h] && dist[h] >= n) mark |= anc[h];
+    if (good[h] && ts.dist[h] >= n) mark |= ts.anc[h];
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) mark |= __shfl_xor_sync(0xffffffffu, mark, off);
   // top-down: lowest marked child at each level
   int cur = 0;
   if (lane == 0) s_path[0] = 0;
   for (int k = 1; k <= n; ++k) {
-    const unsigned lo = __ballot_sync(0xffffffffu, par[0] == cur && ((mark >> lane) & 1ull));
-    const unsigned hi = __ballot_sync(0xffffffffu, par[1] == cur && ((mark >> (lane + 32)) & 1ull));
+    const unsigned lo = __ballot_sync(0xffffffffu, ts.par[0] == cur && ((mark >> lane) & 1ull));
+    const unsigned hi = __ballot_sync(0xffffffffu, ts.par[1] == cur && ((mark >> (lane + 32)) & 1ull));
     cur = lo ? (__ffs(lo) - 1) : (__ffs(hi) + 31);
     if (lane == 0) s_path[k] = cur;
   }
   __syncwarp();
   return {n, 0};
+}
+
+// Both phases at once (the stand-alone accept walk).
+__device__ WalkOut tree_walk_warp(const int32_t *par_row, const int32_t *tok_row, const int32_t *pred_row, int T,
+                                  int max_path, int32_t *s_path) {
+  const TreeShape ts = tree_shape_warp(par_row, tok_row, T);
+  if (ts.bad) return {-1, ts.bad};
+  return tree_walk_finish(ts, pred_row, T, max_path, s_path);
 }
 
 // Writes accept_len, path, out_tokens and new_kv_len of sequence b (warp).
@@ -944,16 +977,21 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
   __shared__ int32_t s_path[65];
   __shared__ int64_t s_src[65], s_dst[65];
   __shared__ int s_n;
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int b = blockIdx.x, Tm = p.tr.T_max;
   const int64_t rb = int64_t(b) * Tm;
   const int T = __ldg(p.tr.tree_len + b);
   const int L = __ldg(p.tr.kv_len + b);
+  // the tree's shape needs no prediction: computed while the argmax grid runs
+  const bool lens_ok = T >= 1 && T <= Tm && L >= 0 && L <= p.kv.capacity - T;
+  TreeShape ts{};
+  if (threadIdx.x < 32 && lens_ok) ts = tree_shape_warp(p.tr.parent + rb, p.tr.tokens + rb, T);
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (threadIdx.x < 32) {
     WalkOut w{-1, 0};
     if (T < 1 || T > Tm) w.bad = DREAMS_DATA_BAD_TREE_LEN;
     else if (L < 0 || L > p.kv.capacity - T) w.bad = DREAMS_DATA_BAD_KV_LEN;
-    else w = tree_walk_warp(p.tr.parent + rb, p.tr.tokens + rb, p.pred + rb, T, p.max_path, s_path);
+    else if (ts.bad) w.bad = ts.bad;
+    else w = tree_walk_finish(ts, p.pred + rb, T, p.max_path, s_path);
     if (w.bad) {
       w.n = -1;
       if (threadIdx.x == 0) flag(p.status, w.bad);
