@@ -533,7 +533,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     }
   } else if (warp == MMA_WARP) {
     // ---------------- MMA issuer
-    if (lane == 0 && tree_ok) {
+    if (lane == 0) {  // a malformed tree stops it through the abort flag
       // Base descriptors: an operand's descriptor is its base plus its byte
       // offset / 16 (the address field holds bits 4-17 of a shared-memory
       // address below 256 KB, so the addition never carries out of it); each
