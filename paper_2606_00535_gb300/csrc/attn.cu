@@ -311,28 +311,6 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     if (pi < p.pages_per_seq) pn_pre[0] = __ldg(prow + pi);
     if (pi + 1 < p.pages_per_seq) pn_pre[1] = __ldg(prow + pi + 1);
   }
-  const bool reporter = (rb == 0 && split == 0 && g == 0);
-  const int T = __ldg(p.tree_len + b);
-  const int L = __ldg(p.kv_len + b);
-  if (T < 1 || T > p.T_max) {
-    if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_TREE_LEN);
-    return;
-  }
-  const int total = key_total(p, L, T);
-  if (L < 0 || total > p.capacity || total < 1) {
-    if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_KV_LEN);
-    return;
-  }
-  const int nsplit_b = (total + p.chunk - 1) / p.chunk;
-  const int t0 = rb * p.TB;  // first tree node of the row block
-  if (split >= nsplit_b || t0 >= T) return;
-  // keys any row of the block may attend: a causal block stops after its last row's own slot
-  const int kend = p.mode == ATTN_CAUSAL ? L + ::min(T, t0 + p.TB) : total;
-  if (split * p.chunk >= kend) return;
-  const int rows_blk = ::min(p.TB, T - t0) * p.G;  // real query rows of this CTA
-  // softmax warps whose 32 rows hold at least one real query row
-  const int n_act = ::min(4, (rows_blk + 31) / 32);
-
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t q_s = smem_base;
   auto k_s = [&](int st) { return smem_base + Q_BYTES + uint32_t(st) * KV_TILE; };
@@ -341,8 +319,16 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const uint32_t vf0 = smem_u32(&bar_vf[0]), ve0 = smem_u32(&bar_ve[0]);
   const uint32_t bs0 = smem_u32(&bar_s[0]), bp0 = smem_u32(&bar_p[0]);
   const uint32_t bq = smem_u32(&bar_q), bdrain = smem_u32(&bar_drain);
+  const int t0 = rb * p.TB;  // first tree node of the row block
+  const int c0 = split * p.chunk;
 
-  if (tid == TMA_WARP * 32) {
+  // With a contiguous cache and the pair known from the grid index, the Q
+  // block and the first K tile have known coordinates before the lengths
+  // arrive: the producer sets up the copy barriers and issues both at once.
+  // A CTA that then turns out to have nothing to do waits for them to land
+  // before it exits.
+  const bool early = !P.paged && p.order == nullptr && !p.rank;
+  auto init_copy_barriers = [&]() {
     for (int i = 0; i < NK; ++i) {
       tc::mbar_init(kf0 + 8 * i, 1);
       tc::mbar_init(ke0 + 8 * i, 1);
@@ -351,14 +337,70 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       tc::mbar_init(vf0 + 8 * i, 1);
       tc::mbar_init(ve0 + 8 * i, 1);
     }
+    tc::mbar_init(bq, 1);
+    s_zero = 0;
+  };
+  auto issue_q = [&]() {
+    tc::prefetch_tmap(&P.tmap_q);
+    tc::prefetch_tmap(&P.tmap_k);
+    tc::prefetch_tmap(&P.tmap_v);
+    // the Q rows of the block: G heads x TB nodes per 64-column region
+    // (nodes past T_max read as zeros; the transaction counts the full box)
+    tc::mbar_arrive_expect_tx(bq, uint32_t(NR * p.G * p.TB * 128));
+#pragma unroll
+    for (int r = 0; r < NR; ++r) tc::tma_load_5d(q_s + r * Q_REGION, &P.tmap_q, bq, r * 64, 0, g, t0, b);
+  };
+  if (early && tid == TMA_WARP * 32) {
+    init_copy_barriers();
+    tc::fence_barrier_init();
+    issue_q();
+    tc::mbar_arrive_expect_tx(kf0, KV_TILE);
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+      tc::tma_load_4d(k_s(0) + r * KV_REGION, &P.tmap_k, kf0, r * 64, g, c0, b);
+      tc::tma_load_4d(k_s(0) + r * KV_REGION + 8192, &P.tmap_k, kf0, r * 64, g, c0 + 64, b);
+    }
+  }
+  auto leave = [&]() {
+    if (early && tid == TMA_WARP * 32) {
+      tc::mbar_wait(bq, 0, &s_zero);
+      tc::mbar_wait(kf0, 0, &s_zero);
+    }
+  };
+
+  const bool reporter = (rb == 0 && split == 0 && g == 0);
+  const int T = __ldg(p.tree_len + b);
+  const int L = __ldg(p.kv_len + b);
+  if (T < 1 || T > p.T_max) {
+    if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_TREE_LEN);
+    leave();
+    return;
+  }
+  const int total = key_total(p, L, T);
+  if (L < 0 || total > p.capacity || total < 1) {
+    if (reporter && tid == 0) flag(p.status, DREAMS_DATA_BAD_KV_LEN);
+    leave();
+    return;
+  }
+  const int nsplit_b = (total + p.chunk - 1) / p.chunk;
+  // keys any row of the block may attend: a causal block stops after its last row's own slot
+  const int kend = p.mode == ATTN_CAUSAL ? L + ::min(T, t0 + p.TB) : total;
+  if (split >= nsplit_b || t0 >= T || c0 >= kend) {
+    leave();
+    return;
+  }
+  const int rows_blk = ::min(p.TB, T - t0) * p.G;  // real query rows of this CTA
+  // softmax warps whose 32 rows hold at least one real query row
+  const int n_act = ::min(4, (rows_blk + 31) / 32);
+
+  if (tid == TMA_WARP * 32) {
+    if (!early) init_copy_barriers();
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(bs0 + 8 * i, 1);
       tc::mbar_init(bp0 + 8 * i, 32 * n_act);
     }
-    tc::mbar_init(bq, 1);
     tc::mbar_init(bdrain, 1);
     s_abort = 0;
-    s_zero = 0;
     s_flag = 0;
     tc::fence_barrier_init();
   }
@@ -371,7 +413,6 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   tc::fence_after_sync();
   const uint32_t tmem = s_tmem;
 
-  const int c0 = split * p.chunk;
   const int c1 = ::min(c0 + p.chunk, kend);
   const int ntiles = (c1 - c0 + KT - 1) / KT;
   volatile int *abort_flag = &s_abort;
@@ -448,14 +489,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   if (warp == TMA_WARP) {
     // ---------------- TMA producer
     if (lane == 0) {
-      tc::prefetch_tmap(&P.tmap_q);
-      tc::prefetch_tmap(&P.tmap_k);
-      tc::prefetch_tmap(&P.tmap_v);
-      // the Q rows of the block: G heads x TB nodes per 64-column region
-      // (nodes past T_max read as zeros; the transaction counts the full box)
-      tc::mbar_arrive_expect_tx(bq, uint32_t(NR * p.G * p.TB * 128));
-#pragma unroll
-      for (int r = 0; r < NR; ++r) tc::tma_load_5d(q_s + r * Q_REGION, &P.tmap_q, bq, r * 64, 0, g, t0, b);
+      if (!early) issue_q();  // (else already issued, with K_0)
       // raw page-table entries of the two 64-slot halves of tile j
       const int32_t *prow = P.paged ? p.page_table + int64_t(b) * p.pages_per_seq : nullptr;
       auto fetch = [&](int j, int &e0, int &e1) {
@@ -478,6 +512,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       int ring[CRD][2];
       int pn0 = pn_pre[0], pn1 = pn_pre[1];  // tile 0 (loaded at the start)
       int nk = 0, nv = 0;  // tiles issued into each ring
+      if (early) {  // K_0 went out at the start
+        ring[0][0] = ring[0][1] = b;
+        nk = 1;
+      }
       uint32_t idle = 0;
       uint64_t t_idle = 0;
       while (nv < ntiles && !*abort_flag) {
