@@ -49,13 +49,12 @@
 //                       signals P_j it waits for V_j and K_{j+2} to land, so
 //                       that the MMA thread needs no other wait. Warps whose
 //                       rows are all padding sit out.
-// At the end the two warpgroups combine their (m, l, O) by log-sum-exp into a
-// swizzled staging copy in the idle shared-memory rings, and all 256 threads
-// write it out in row order (16-byte coalesced stores): the output, or the
-// split partials that a merge kernel (chained by programmatic dependent
-// launch) combines. Every mbarrier wait is bounded (2 s); on a timeout the CTA
-// flags DREAMS_DATA_TIMEOUT, drains its copies and MMAs, frees its TMEM and
-// exits. The workspace holds no state between calls.
+// At the end the two warpgroups combine their (m, l, O) by log-sum-exp and
+// each thread writes its row's half of the columns with 16-byte stores: the
+// output, or the split partials that a merge kernel (chained by programmatic
+// dependent launch) combines. Every mbarrier wait is bounded (2 s); on a
+// timeout the CTA flags DREAMS_DATA_TIMEOUT, drains its copies and MMAs, frees
+// its TMEM and exits. The workspace holds no state between calls.
 #include <cuda.h>
 #include <limits.h>
 #include <math.h>
@@ -800,11 +799,10 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     sm_ok = ok;
   }
 
-  // ---- epilogue: the two warpgroups combine their (m, l, O) into a swizzled
-  // staging copy (row-major, 16-byte chunks XOR-ed with row & 7 so that the
-  // 32 rows of a warp hit distinct banks); then all 256 threads copy it out in
-  // row order. The rings are idle once every MMA has completed: the staging
-  // copy takes the Q region and the K ring, (m, l) the last V stage.
+  // ---- epilogue: the two warpgroups combine their (m, l, O) by log-sum-exp
+  // ((m, l) pass through the last V stage, idle once every MMA has completed);
+  // each thread then writes its row's half of the columns straight to global
+  // memory in 16-byte stores: the output, or the split partials.
   if (warp < 8) {
     const bool act = (warp & 3) < n_act && tree_ok;
     // the output directly, unless the block's keys span several splits
@@ -827,8 +825,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const float Ls = ca * a.y + cb * c.y;
       const uint32_t lanes = tmem + (uint32_t(32 * (warp & 3)) << 16);
       const float inv = direct ? 1.f / Ls : 1.f;
-      const uint32_t rbytes = direct ? D * 2 : D * 4;
-      const uint32_t srow = smem_base + row * rbytes;
+      const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + (row - (t_row - t0) * p.G);
 #pragma unroll 1
       for (int c4 = 0; c4 < D / 64; ++c4) {
         const int col = wg * (D / 2) + c4 * 32;
@@ -843,26 +840,17 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           const float vb = cb != 0.f ? cb * __uint_as_float(ob[e]) : 0.f;
           o[e] = (va + vb) * inv;
         }
+        if (!real_row) continue;
         if (direct) {
+          uint4 *dst = reinterpret_cast<uint4 *>(p.out + orow * D + col);
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int ch = col / 8 + e;  // 16-byte chunk of 8 bf16
-            const uint32_t dst = srow + ((ch >> 3) << 7) + (((ch & 7) ^ (row & 7)) << 4);
-            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst),
-                         "r"(pack_bf16x2(o[8 * e + 0], o[8 * e + 1])), "r"(pack_bf16x2(o[8 * e + 2], o[8 * e + 3])),
-                         "r"(pack_bf16x2(o[8 * e + 4], o[8 * e + 5])), "r"(pack_bf16x2(o[8 * e + 6], o[8 * e + 7]))
-                         : "memory");
-          }
+          for (int e = 0; e < 4; ++e)
+            dst[e] = make_uint4(pack_bf16x2(o[8 * e + 0], o[8 * e + 1]), pack_bf16x2(o[8 * e + 2], o[8 * e + 3]),
+                                pack_bf16x2(o[8 * e + 4], o[8 * e + 5]), pack_bf16x2(o[8 * e + 6], o[8 * e + 7]));
         } else {
+          float4 *dst = reinterpret_cast<float4 *>(p.ws_o + (slot + row) * D + col);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int ch = col / 4 + e;  // 16-byte chunk of 4 floats
-            const uint32_t dst = srow + ((ch >> 3) << 7) + (((ch & 7) ^ (row & 7)) << 4);
-            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(__float_as_uint(o[4 * e + 0])),
-                         "r"(__float_as_uint(o[4 * e + 1])), "r"(__float_as_uint(o[4 * e + 2])),
-                         "r"(__float_as_uint(o[4 * e + 3]))
-                         : "memory");
-          }
+          for (int e = 0; e < 8; ++e) dst[e] = make_float4(o[4 * e], o[4 * e + 1], o[4 * e + 2], o[4 * e + 3]);
         }
       }
       if (wg == 0 && real_row) {
@@ -874,40 +862,12 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           if (ca != 0.f) Wt += ca * (s_w[row] + (a.x - M) * a.y);
           if (cb != 0.f) Wt += cb * (s_w[ROWS + row] + (c.x - M) * c.y);
         }
-        const int64_t orow = (int64_t(b) * p.T_max + t_row) * p.Hq + g * p.G + (row - (t_row - t0) * p.G);
         if (direct) {
           if (p.lse != nullptr) p.lse[orow] = (M + log2f(Ls)) * LN2;
           if (ENT && p.ent != nullptr) p.ent[orow] = logf(Ls) - LN2 * Wt / Ls;
         } else {
           p.ws_ml[slot + row] = make_float2(Ls > 0.f ? M : -INFINITY, Ls);
           if (ENT) p.ws_w[slot + row] = Ls > 0.f ? Wt : 0.f;
-        }
-      }
-    }
-    named_sync(3, 256);
-    if (tree_ok && !*abort_flag) {
-      if (direct) {
-        constexpr int CH = D / 8;
-        for (int i = tid; i < rows_blk * CH; i += 256) {
-          const int r = i / CH, ch = i - r * CH;
-          uint4 v;
-          asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];"
-                       : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                       : "r"(smem_base + r * (D * 2) + ((ch >> 3) << 7) + (((ch & 7) ^ (r & 7)) << 4)));
-          const int tn = r / p.G;
-          const int64_t orow = (int64_t(b) * p.T_max + t0 + tn) * p.Hq + g * p.G + (r - tn * p.G);
-          *reinterpret_cast<uint4 *>(p.out + orow * D + ch * 8) = v;
-        }
-      } else {
-        constexpr int CH = D / 4;
-        float4 *dst = reinterpret_cast<float4 *>(p.ws_o + slot * D);
-        for (int i = tid; i < rows_blk * CH; i += 256) {
-          const int r = i / CH, ch = i - r * CH;
-          float4 v;
-          asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                       : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                       : "r"(smem_base + r * (D * 4) + ((ch >> 3) << 7) + (((ch & 7) ^ (r & 7)) << 4)));
-          dst[i] = v;
         }
       }
     }
