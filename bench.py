@@ -25,6 +25,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -62,6 +63,12 @@ def parse():
                     help="untimed steps run while the clock sampler starts (0 under a profiler)")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch every call from Python in the timed loop instead of replaying CUDA graphs")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the attention and verify-step timings of the other workloads (tiny, llava7b, "
+                         "qwen2vl7b, long13b)")
+    ap.add_argument("--clock-log", default=None,
+                    help="keep the nvidia-smi clock samples of the timed region in this CSV file (default: a "
+                         "temporary file, removed afterwards)")
     ap.add_argument("--flush-l2", action="store_true",
                     help="before every timed step (outside its events) write a buffer twice the size of L2, then "
                          "read another as large, so that L2 holds only clean unrelated lines; average the per-step "
@@ -130,14 +137,19 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, path=None):
         self.proc = None
         self.gpu = gpu_index
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+        self.keep = path is not None
+        if path is None:
+            fd, path = tempfile.mkstemp(prefix=f"dreams_clocks_gpu{gpu_index}_", suffix=".csv")
+            os.close(fd)
+        self.path = path
 
     def start(self):
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            d = os.path.dirname(os.path.abspath(self.path))
+            os.makedirs(d, exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
                                           "--format=csv,noheader,nounits", "-lms", "100"],
@@ -156,7 +168,11 @@ class ClockSampler:
         self.f.close()
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path):
+        with open(self.path) as f:
+            lines = f.readlines()
+        if not self.keep:
+            os.unlink(self.path)
+        for line in lines:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
@@ -190,6 +206,77 @@ def max_over_ranks(x: float, device) -> float:
     t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+# ---------------------------------------------------------------- per-workload timings
+def time_workload(dreams, dev, name: str, K: int, status, barrier) -> dict:
+    """Attention and verification-tail times of one workload, the same calls as
+    the headline step: two input copies, each copy's two calls captured as
+    CUDA graphs, CUDA events on the launching stream. These workloads fit in
+    L2, so before every step (outside its events) a buffer twice the size of
+    L2 is written, then another as large as L2 read; the per-step times are
+    averaged."""
+    w = W.make(name)
+    copies = []
+    for _ in range(2):
+        c = {"q": w.q.to(dev), "k": w.k.to(dev), "v": w.v.to(dev),
+             "pt": None if w.page_table is None else w.page_table.to(dev), "logits": w.logits.to(dev)}
+        c["kv"] = dreams.KVCache(c["k"], c["v"], c["pt"])
+        c["tree"] = dreams.Tree(w.parent.to(dev), w.tokens.to(dev), w.tree_len.to(dev), w.kv_len.to(dev))
+        c["out"] = torch.empty_like(c["q"])
+        c["outs"] = (torch.empty(w.B, dtype=torch.int32, device=dev),
+                     torch.empty((w.B, w.max_path), dtype=torch.int32, device=dev),
+                     torch.empty((w.B, w.max_path), dtype=torch.int32, device=dev),
+                     torch.empty(w.B, dtype=torch.int32, device=dev))
+        copies.append(c)
+    n_ws = dreams.tree_verify_attn_workspace_size(copies[0]["kv"], copies[0]["tree"], w.Hq)
+    ws_attn = torch.zeros(max(16, n_ws), dtype=torch.uint8, device=dev)
+    ws_step = torch.zeros(dreams.verify_step_workspace_size(copies[0]["tree"], w.V), dtype=torch.uint8, device=dev)
+
+    def attn_call(c):
+        dreams.tree_verify_attn(c["q"], c["kv"], c["tree"], w.scale, out=c["out"],
+                                workspace=ws_attn if n_ws else None, status=status)
+
+    def step_call(c):
+        dreams.verify_step(c["logits"], c["tree"], c["kv"], w.max_path, outputs=c["outs"], workspace=ws_step,
+                           status=status)
+
+    for i in range(4):
+        attn_call(copies[i % 2])
+        step_call(copies[i % 2])
+    torch.cuda.synchronize(dev)
+    graphs = []
+    for c in copies:
+        ga, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(ga):
+            attn_call(c)
+        with torch.cuda.graph(gs):
+            step_call(c)
+        graphs.append((ga, gs))
+    stream = torch.cuda.current_stream(dev)
+    flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    flush_read = torch.zeros(L2_BYTES // 2, dtype=torch.float32, device=dev)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    for i in range(2):
+        graphs[i][0].replay()
+        graphs[i][1].replay()
+    barrier()
+    for i in range(K):
+        flush_buf.fill_(i & 255)
+        flush_read.sum()
+        evs[i][0].record(stream)
+        graphs[i % 2][0].replay()
+        evs[i][1].record(stream)
+        graphs[i % 2][1].replay()
+        evs[i][2].record(stream)
+    barrier()
+    a_us = sum(e[0].elapsed_time(e[1]) for e in evs) / K * 1000.0
+    v_us = sum(e[1].elapsed_time(e[2]) for e in evs) / K * 1000.0
+    ab, gb = attn_bytes(w), argmax_bytes(w)
+    return {"workload": w.spec.description, "attn_us": round(a_us, 2), "attn_bytes": ab,
+            "attn_GBps": round(ab / (a_us * 1e-6) / 1e9, 1), "verify_us": round(v_us, 2), "argmax_bytes": gb,
+            "verify_argmax_GBps": round(gb / (v_us * 1e-6) / 1e9, 1), "step_us": round(a_us + v_us, 2),
+            "launch": "cuda-graph replay", "l2": "flushed before every step (outside its events)", "steps": K}
 
 
 # ---------------------------------------------------------------- dreams arm
@@ -293,7 +380,7 @@ def run_dreams(args, rank, world, local):
             graphs = None
             launch_mode = f"eager (graph capture failed: {str(e)[:80]})"
 
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(local, None if args.clock_log is None else args.clock_log.replace("{rank}", str(rank)))
     clocks.start()
     t_load = time.time()  # keep the GPU busy ~1 s so the sampler sees the clocks under this load
     while time.time() - t_load < args.load_seconds:
@@ -539,6 +626,14 @@ def run_dreams(args, rank, world, local):
         }
         del kvs, qx, qp
 
+    per_config = None
+    if not args.no_per_config:
+        per_config = {}
+        for name in [s.name for s in W.SPECS if s.name != args.config]:
+            per_config[name] = time_workload(dreams, dev, name, max(3, min(K, 50)), status, barrier)
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item()):#x} (per-workload timings)")
+
     ab, gb = attn_bytes(w), argmax_bytes(w)
     attn_avg_ms = sum(attn_ms) / K
     tail_avg_ms = sum(tail_ms) / K
@@ -571,6 +666,11 @@ def run_dreams(args, rank, world, local):
     if modes is not None:
         modes["cross_attention"]["frac_measured_hbm"] = round(modes["cross_attention"]["GBps"] / peak, 4)
         kernels.update(modes)
+    if per_config is not None:
+        for rec in per_config.values():
+            rec["attn_frac_measured_hbm"] = round(rec["attn_GBps"] / peak, 4)
+            rec["verify_frac_measured_hbm"] = round(rec["verify_argmax_GBps"] / peak, 4)
+        kernels["per_config"] = per_config
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

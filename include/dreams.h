@@ -127,12 +127,18 @@ typedef struct dreams_tree {
  *     out[b, t, h, :] = sum_{j in J} softmax_j(scale * <q, K[b, j, g]>) V[b, j, g, :]
  *     lse[b, t, h]    = log sum_{j in J} exp(scale * <q, K[b, j, g]>)
  * Hq must be a multiple of kv->Hkv with at most 128 query heads per KV head.
- * q, out: bf16 [B, T_max, Hq, D] (16-byte aligned). lse: f32 [B, T_max, Hq]
- * or NULL. Rows t >= tree_len[b] of out and lse are left untouched, and so are
- * all rows of a sequence with bad data. layer selects the cache
- * (0 <= layer < kv->n_layers). scale must be finite and > 0. Accumulation is
- * fp32 (the probabilities enter the PV product as bf16); the output is
- * rounded to bf16 once.
+ * q: bf16, element (b, t, h, d) at q[b * q_stride_b + t * q_stride_t + h * D + d]:
+ * each token's Hq head rows are dense, tokens and sequences are strided, so Q
+ * may be a view into a fused QKV projection output (e.g. [B, T, 3, Hq, D]:
+ * q_stride_t = 3 Hq D, q_stride_b = T_max q_stride_t). Both strides are in
+ * elements, at least Hq * D, multiples of 8 (16 bytes) and below 2^38;
+ * q_stride_b is ignored when B == 1. out: bf16 [B, T_max, Hq, D], dense.
+ * q and out 16-byte aligned. lse: f32 [B, T_max, Hq] or NULL. Rows
+ * t >= tree_len[b] of out and lse are left untouched, and so are all rows of a
+ * sequence with bad data, and the rows a call that flags DREAMS_DATA_TIMEOUT
+ * did not finish. layer selects the cache (0 <= layer < kv->n_layers). scale
+ * must be finite and > 0. Accumulation is fp32 (the probabilities enter the
+ * PV product as bf16); the output is rounded to bf16 once.
  */
 size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const dreams_tree_t *tree,
                                               int32_t Hq);
@@ -142,7 +148,8 @@ size_t dreams_tree_verify_attn_workspace_size(const dreams_kv_cache_t *kv, const
  * attention, a merge of the KV splits when the cache is split); 0 for shapes
  * the call rejects. */
 int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv, const dreams_tree_t *tree, int32_t Hq);
-dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+dreams_status_t dreams_tree_verify_attn(const void *q, int64_t q_stride_b, int64_t q_stride_t,
+                                        const dreams_kv_cache_t *kv, int32_t layer,
                                         const dreams_tree_t *tree, int32_t Hq, float scale, void *out,
                                         float *lse, void *workspace, size_t workspace_bytes,
                                         int32_t *status_word, dreams_stream_t stream);
@@ -159,8 +166,9 @@ dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *
  *   DREAMS_ATTN_CAUSAL query t attends slots 0 .. kv_len[b] + t: its own slot
  *                      is kv_len[b] + t (prefill of a layer, A = softmax(QK^T /
  *                      sqrt(z)) of Sec. 3.3).
- * q, out: bf16 [B, T_max, Hq, D]; q_len[b] in [1, T_max] query rows are
- * computed (T_max <= 2^20); kv as for dreams_tree_verify_attn (FULL needs
+ * q (strided as for dreams_tree_verify_attn), out: bf16 [B, T_max, Hq, D];
+ * q_len[b] in [1, T_max] query rows are computed (T_max <= 2^20); kv as for
+ * dreams_tree_verify_attn (FULL needs
  * kv_len >= 1, CAUSAL kv_len + q_len <= capacity). lse and entropy: f32
  * [B, T_max, Hq] or NULL. entropy[b][t][h] = -sum_j a_j ln a_j over the row's
  * attention weights a (nats); the average over rows and heads is AE(l) of
@@ -171,7 +179,8 @@ dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *
 #define DREAMS_ATTN_CAUSAL 2
 size_t dreams_attention_workspace_size(const dreams_kv_cache_t *kv, int32_t B, int32_t T_max, int32_t Hq,
                                        int32_t mode, int32_t want_entropy);
-dreams_status_t dreams_attention(const void *q, const dreams_kv_cache_t *kv, int32_t layer, const int32_t *q_len,
+dreams_status_t dreams_attention(const void *q, int64_t q_stride_b, int64_t q_stride_t, const dreams_kv_cache_t *kv,
+                                 int32_t layer, const int32_t *q_len,
                                  const int32_t *kv_len, int32_t B, int32_t T_max, int32_t Hq, float scale,
                                  int32_t mode, void *out, float *lse, float *entropy, void *workspace,
                                  size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream);
@@ -309,7 +318,8 @@ dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dt
  * the indices and resets the slots. The workspace holds the slots: zero-fill
  * it once when it is allocated; every call leaves it zero-filled. A wait that
  * times out inside the GEMM flags DREAMS_DATA_TIMEOUT in status_word (may be
- * NULL).
+ * NULL); the indices of such a call are then unreliable, except that rows no
+ * tile reached are left untouched.
  */
 size_t dreams_lm_head_argmax_workspace_size(int64_t rows);
 dreams_status_t dreams_lm_head_argmax(const void *hidden, int64_t rows, int64_t hidden_dim, int64_t ld_hidden,
@@ -366,6 +376,29 @@ dreams_status_t dreams_visual_importance(const void *attn, dreams_dtype_t dtype,
 #define DREAMS_NOALLOC_ARGMAX_MAX_ROWS 16384
 dreams_status_t dreams_vocab_argmax_noalloc(const void *logits, dreams_dtype_t dtype, int64_t rows, int64_t V,
                                             int64_t row_stride, int32_t *out_idx, dreams_stream_t stream);
+
+/*
+ * Test hook for the bounded pipeline waits of the tcgen05 kernels; not for
+ * production use. The paper has no counterpart: every wait of these kernels
+ * on its own copy or MMA pipeline gives up after a limit instead of hanging
+ * the GPU, and this hook lets a test make such a wait run out without any
+ * fault. While stall_at >= 0, every later launch of the kernels selected by
+ * `kernels` (DREAMS_TEST_ATTENTION: dreams_tree_verify_attn and
+ * dreams_attention; DREAMS_TEST_LM_HEAD: dreams_lm_head_argmax) withholds the
+ * TMA copies of each CTA from its stall_at-th K tile (attention) or k-block
+ * (LM head, counted over the CTA's tiles) on, waiting instead on a barrier
+ * that nothing arrives on, and every pipeline wait gives up after
+ * wait_limit_ns (1 us .. 2 s) instead of 2 s. The kernels then flag
+ * DREAMS_DATA_TIMEOUT, wait for the copies and MMAs they did issue, free
+ * their tensor memory and exit; output rows they did not finish are left
+ * untouched (attention), or unreliable (LM head; rows no tile reached are
+ * untouched). stall_at < 0 restores normal operation (the other arguments
+ * are then ignored). The setting is process-wide and read at launch, so a
+ * CUDA graph keeps the setting it was captured with.
+ */
+#define DREAMS_TEST_ATTENTION 1
+#define DREAMS_TEST_LM_HEAD 2
+dreams_status_t dreams_test_set_stall(int32_t kernels, int32_t stall_at, int64_t wait_limit_ns);
 
 const char *dreams_status_string(dreams_status_t status);
 int32_t dreams_version(void);

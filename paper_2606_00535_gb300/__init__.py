@@ -35,6 +35,7 @@ NOALLOC_ARGMAX_MAX_ROWS = 16384
 F32, BF16 = 0, 1
 DATA_BAD_PARENT, DATA_BAD_TREE_LEN, DATA_BAD_KV_LEN, DATA_BAD_PAGE, DATA_BAD_PATH = 1, 2, 4, 8, 16
 DATA_TIMEOUT = 0x20  # a kernel gave up waiting on its own pipeline
+TEST_ATTENTION, TEST_LM_HEAD = 1, 2  # kernel families of test_set_stall
 
 
 class DreamsError(RuntimeError):
@@ -78,7 +79,8 @@ def _lib() -> ctypes.CDLL:
                 sig = {
                     "dreams_tree_verify_attn_workspace_size": (sz, [pkv, ptr, i32]),
                     "dreams_tree_verify_attn_launches": (i32, [pkv, ptr, i32]),
-                    "dreams_tree_verify_attn": (ctypes.c_int, [p, pkv, i32, ptr, i32, f32, p, p, p, sz, p, p]),
+                    "dreams_tree_verify_attn": (ctypes.c_int, [p, i64, i64, pkv, i32, ptr, i32, f32, p, p, p, sz, p,
+                                                               p]),
                     "dreams_vocab_argmax_workspace_size": (sz, [i64, i64]),
                     "dreams_vocab_argmax": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p, sz, p]),
                     "dreams_accept_path": (ctypes.c_int, [p, ptr, i32, p, p, p, p, p, p]),
@@ -88,8 +90,8 @@ def _lib() -> ctypes.CDLL:
                                                           p, p, sz, p, p]),
                     "dreams_vocab_argmax_noalloc": (ctypes.c_int, [p, ctypes.c_int, i64, i64, i64, p, p]),
                     "dreams_attention_workspace_size": (sz, [pkv, i32, i32, i32, i32, i32]),
-                    "dreams_attention": (ctypes.c_int, [p, pkv, i32, p, p, i32, i32, i32, f32, i32, p, p, p, p, sz,
-                                                        p, p]),
+                    "dreams_attention": (ctypes.c_int, [p, i64, i64, pkv, i32, p, p, i32, i32, i32, f32, i32, p, p,
+                                                        p, p, sz, p, p]),
                     "dreams_lm_head_argmax_workspace_size": (sz, [i64]),
                     "dreams_lm_head_argmax": (ctypes.c_int, [p, i64, i64, i64, p, i64, i64, p, p, p, sz, p, p]),
                     "dreams_visual_importance_workspace_size": (sz, [i64, i64, i64, i64]),
@@ -100,6 +102,7 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step_sampled_workspace_size": (sz, [ptr, i64]),
                     "dreams_verify_step_sampled": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, f32, p,
                                                                   p, p, p, p, p, p, sz, p, p]),
+                    "dreams_test_set_stall": (ctypes.c_int, [i32, i32, i64]),
                     "dreams_status_string": (ctypes.c_char_p, [ctypes.c_int]),
                     "dreams_version": (i32, []),
                     "dreams_last_cuda_error": (i32, []),
@@ -126,14 +129,48 @@ def _ptr(t: Optional[torch.Tensor]):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
-def _stream(stream) -> ctypes.c_void_p:
-    s = torch.cuda.current_stream() if stream is None else stream
+def _stream(stream, dev: torch.device) -> ctypes.c_void_p:
+    """The given stream, or the current stream of the tensors' device ``dev``."""
+    s = torch.cuda.current_stream(dev) if stream is None else stream
+    if s.device != dev:
+        raise ValueError(f"stream is on {s.device}, the tensors on {dev}")
     return ctypes.c_void_p(s.cuda_stream)
 
 
 def _check(name: str, st: int):
     if st != OK:
         raise DreamsError(name, st)
+
+
+def _call(name: str, dev: torch.device, *args) -> None:
+    """Calls the C entry point with the tensors' device current (the library
+    runs on the current CUDA device) and raises on a non-OK status."""
+    if dev.type != "cuda":
+        raise ValueError(f"{name}: tensors must be on a CUDA device, got {dev}")
+    with torch.cuda.device(dev):
+        st = getattr(_lib(), name)(*args)
+    _check(name, st)
+
+
+def _rows_view(logits: torch.Tensor) -> torch.Tensor:
+    """[rows, V] view of ``logits`` (no copy) with contiguous rows."""
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    V = int(logits.shape[-1])
+    try:
+        x = logits if logits.dim() == 2 else logits.view(-1, V)
+    except RuntimeError as e:
+        raise ValueError("logits' leading dimensions must flatten without a copy") from e
+    if x.stride(-1) != 1:
+        raise ValueError("logits rows must be contiguous")
+    return x
+
+
+def _need_out(out: torch.Tensor, name: str, dtype, dev, numel: int) -> torch.Tensor:
+    _need(out, name, dtype, dev)
+    if out.numel() < numel:
+        raise ValueError(f"{name} holds {out.numel()} elements, {numel} are written")
+    return out
 
 
 def _need(t: torch.Tensor, name: str, dtype, dev) -> torch.Tensor:
@@ -241,53 +278,63 @@ VERIFY_STEP_LAUNCHES = 2
 VERIFY_STEP_SAMPLED_LAUNCHES = 3  # draw statistics, draw selection, walk + compaction  # dreams_verify_step: the argmax, then the walk and compaction
 
 
+def _q_strides(q: torch.Tensor) -> Tuple[int, int]:
+    """(sequence stride, token stride) in elements of a bf16 [B, T, Hq, D]
+    query tensor whose head rows are dense (a view into a fused QKV output
+    qualifies)."""
+    if not isinstance(q, torch.Tensor) or q.dtype != torch.bfloat16 or q.dim() != 4:
+        raise TypeError("q must be a 4-D bfloat16 tensor [B, T, Hq, D]")
+    if q.stride(3) != 1 or q.stride(2) != q.shape[3]:
+        raise ValueError("q's head rows must be dense (strides [.., .., D, 1])")
+    return int(q.stride(0)), int(q.stride(1))
+
+
 def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, layer: int = 0,
                      out: Optional[torch.Tensor] = None, lse: Optional[torch.Tensor] = None,
                      want_lse: bool = False, workspace: Optional[torch.Tensor] = None,
                      status: Optional[torch.Tensor] = None, stream=None):
     """Tree-masked attention of the tree tokens' queries ``q`` (bf16
-    [B, T_max, Hq, D]) over the cache. Returns (out, lse or None)."""
+    [B, T_max, Hq, D], head rows dense, tokens and sequences may be strided)
+    over the cache. Returns (out, lse or None); out is dense."""
     dev = q.device
-    _need(q, "q", torch.bfloat16, dev)
+    sb, stt = _q_strides(q)
     Hq = int(q.shape[2])
     if out is None:
-        out = torch.empty_like(q)
+        out = torch.empty(tuple(q.shape), dtype=torch.bfloat16, device=dev)
     _need(out, "out", torch.bfloat16, dev)
+    if tuple(out.shape) != tuple(q.shape):
+        raise ValueError("out must have q's shape")
     if lse is None and want_lse:
         lse = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
     if lse is not None:
         _need(lse, "lse", torch.float32, dev)
+        if tuple(lse.shape) != tuple(q.shape[:3]):
+            raise ValueError("lse must be [B, T_max, Hq]")
     need = tree_verify_attn_workspace_size(kv, tree, Hq)
     if workspace is None:
         workspace = _workspace("attn", need, dev, stream)
-    st = _lib().dreams_tree_verify_attn(
-        _ptr(q), ctypes.byref(kv._c), layer, ctypes.byref(tree._c), Hq, float(scale), _ptr(out), _ptr(lse),
-        _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
-        _ptr(status), _stream(stream))
-    _check("dreams_tree_verify_attn", st)
+    _call("dreams_tree_verify_attn", dev,
+          _ptr(q), sb, stt, ctypes.byref(kv._c), layer, ctypes.byref(tree._c), Hq, float(scale), _ptr(out),
+          _ptr(lse), _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
+          _ptr(status), _stream(stream, dev))
     return out, lse
 
 
 def vocab_argmax(logits: torch.Tensor, out: Optional[torch.Tensor] = None,
                  workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
     """Row-wise argmax of a 2-D (or flattened leading dims) f32 / bf16 tensor."""
-    if logits.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("logits must be float32 or bfloat16")
-    V = int(logits.shape[-1])
-    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
-    if x.stride(-1) != 1:
-        raise ValueError("logits rows must be contiguous")
-    rows = int(x.shape[0])
+    x = _rows_view(logits)
+    rows, V = int(x.shape[0]), int(x.shape[1])
+    dev = logits.device
     if out is None:
-        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=logits.device)
-    _need(out, "out", torch.int32, logits.device)
+        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=dev)
+    _need_out(out, "out", torch.int32, dev, rows)
     need = int(_lib().dreams_vocab_argmax_workspace_size(rows, V))
     if workspace is None:
-        workspace = _workspace("argmax", need, logits.device, stream)
-    st = _lib().dreams_vocab_argmax(
-        _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), _ptr(out),
-        _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
-    _check("dreams_vocab_argmax", st)
+        workspace = _workspace("argmax", need, dev, stream)
+    _call("dreams_vocab_argmax", dev,
+          _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), _ptr(out),
+          _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream, dev))
     return out
 
 
@@ -296,17 +343,16 @@ def vocab_argmax_noalloc(logits: torch.Tensor, out: torch.Tensor, stream=None) -
     allocation, for callers that must not allocate while it runs (see
     ``dreams_vocab_argmax_noalloc`` in include/dreams.h): the library's fixed
     scratch serves at most NOALLOC_ARGMAX_MAX_ROWS rows, and calls that overlap
-    on the GPU race."""
-    if logits.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("logits must be float32 or bfloat16")
-    V = int(logits.shape[-1])
-    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
-    if x.stride(-1) != 1:
-        raise ValueError("logits rows must be contiguous")
-    _need(out, "out", torch.int32, logits.device)
-    st = _lib().dreams_vocab_argmax_noalloc(_ptr(x), F32 if x.dtype == torch.float32 else BF16, int(x.shape[0]), V,
-                                            int(x.stride(0)), _ptr(out), _stream(stream))
-    _check("dreams_vocab_argmax_noalloc", st)
+    on the GPU race. Nothing here allocates: ``logits`` must flatten to
+    [rows, V] as a view, and ``out`` must hold at least ``rows`` int32."""
+    x = _rows_view(logits)
+    rows, V = int(x.shape[0]), int(x.shape[1])
+    if rows > NOALLOC_ARGMAX_MAX_ROWS:
+        raise ValueError(f"{rows} rows exceed the fixed scratch of {NOALLOC_ARGMAX_MAX_ROWS} rows")
+    dev = logits.device
+    _need_out(out, "out", torch.int32, dev, rows)
+    _call("dreams_vocab_argmax_noalloc", dev, _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V,
+          int(x.stride(0)), _ptr(out), _stream(stream, dev))
     return out
 
 
@@ -316,26 +362,22 @@ def vocab_sample(logits: torch.Tensor, temperature: float, uniforms: torch.Tenso
     """One draw per row of a 2-D (or flattened leading dims) f32 / bf16 tensor
     from softmax(row / temperature), by inverse transform with the row's
     uniform (``uniforms``: f32, one per row, on the same device)."""
-    if logits.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("logits must be float32 or bfloat16")
-    V = int(logits.shape[-1])
-    x = logits.reshape(-1, V) if logits.dim() != 2 else logits
-    if x.stride(-1) != 1:
-        raise ValueError("logits rows must be contiguous")
-    rows = int(x.shape[0])
-    _need(uniforms, "uniforms", torch.float32, logits.device)
+    x = _rows_view(logits)
+    rows, V = int(x.shape[0]), int(x.shape[1])
+    dev = logits.device
+    _need(uniforms, "uniforms", torch.float32, dev)
     if uniforms.numel() != rows:
         raise ValueError("uniforms must hold one value per row")
     if out is None:
-        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=logits.device)
-    _need(out, "out", torch.int32, logits.device)
+        out = torch.empty(logits.shape[:-1], dtype=torch.int32, device=dev)
+    _need_out(out, "out", torch.int32, dev, rows)
     need = int(_lib().dreams_vocab_sample_workspace_size(rows, V))
     if workspace is None:
-        workspace = _workspace("sample", need, logits.device, stream)
-    st = _lib().dreams_vocab_sample(
-        _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), float(temperature),
-        _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream))
-    _check("dreams_vocab_sample", st)
+        workspace = _workspace("sample", need, dev, stream)
+    _call("dreams_vocab_sample", dev,
+          _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), float(temperature),
+          _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(),
+          _stream(stream, dev))
     return out
 
 
@@ -349,24 +391,26 @@ def attention(q: torch.Tensor, kv: KVCache, q_len: torch.Tensor, kv_len: torch.T
               status: Optional[torch.Tensor] = None, stream=None):
     """Attention without a tree (ATTN_FULL: the draft's cross-attention to
     target features; ATTN_CAUSAL: a layer's prefill). q: bf16 [B, T_max, Hq,
-    D]. Returns (out, lse, entropy); lse and entropy are None unless asked."""
+    D], head rows dense, tokens and sequences may be strided. Returns (out,
+    lse, entropy); out is dense; lse and entropy are None unless asked."""
     dev = q.device
-    _need(q, "q", torch.bfloat16, dev)
+    sb, stt = _q_strides(q)
     for n, t in (("q_len", q_len), ("kv_len", kv_len)):
         _need(t, n, torch.int32, dev)
     B, T_max, Hq = int(q.shape[0]), int(q.shape[1]), int(q.shape[2])
     if out is None:
-        out = torch.empty_like(q)
+        out = torch.empty(tuple(q.shape), dtype=torch.bfloat16, device=dev)
     _need(out, "out", torch.bfloat16, dev)
+    if tuple(out.shape) != tuple(q.shape):
+        raise ValueError("out must have q's shape")
     lse = torch.empty((B, T_max, Hq), dtype=torch.float32, device=dev) if want_lse else None
     ent = torch.empty((B, T_max, Hq), dtype=torch.float32, device=dev) if want_entropy else None
     need = int(_lib().dreams_attention_workspace_size(ctypes.byref(kv._c), B, T_max, Hq, mode, int(want_entropy)))
     if workspace is None:
         workspace = _workspace("attention", need, dev, stream)
-    st = _lib().dreams_attention(_ptr(q), ctypes.byref(kv._c), layer, _ptr(q_len), _ptr(kv_len), B, T_max, Hq,
-                                 float(scale), mode, _ptr(out), _ptr(lse), _ptr(ent), _ptr(workspace),
-                                 0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
-    _check("dreams_attention", st)
+    _call("dreams_attention", dev, _ptr(q), sb, stt, ctypes.byref(kv._c), layer, _ptr(q_len), _ptr(kv_len), B,
+          T_max, Hq, float(scale), mode, _ptr(out), _ptr(lse), _ptr(ent), _ptr(workspace),
+          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
     return out, lse, ent
 
 
@@ -387,18 +431,17 @@ def lm_head_argmax(hidden: torch.Tensor, weight: torch.Tensor, out: Optional[tor
     dev = hidden.device
     if out is None:
         out = torch.empty(rows, dtype=torch.int32, device=dev)
-    _need(out, "out", torch.int32, dev)
+    _need_out(out, "out", torch.int32, dev, rows)
     if out_max is None and want_max:
         out_max = torch.empty(rows, dtype=torch.float32, device=dev)
     if out_max is not None:
-        _need(out_max, "out_max", torch.float32, dev)
+        _need_out(out_max, "out_max", torch.float32, dev, rows)
     need = int(_lib().dreams_lm_head_argmax_workspace_size(rows))
     if workspace is None:
         workspace = _workspace("lm_head", need, dev, stream)
-    st = _lib().dreams_lm_head_argmax(_ptr(hidden), rows, K, int(hidden.stride(0)), _ptr(weight), V,
-                                      int(weight.stride(0)), _ptr(out), _ptr(out_max), _ptr(workspace),
-                                      0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
-    _check("dreams_lm_head_argmax", st)
+    _call("dreams_lm_head_argmax", dev, _ptr(hidden), rows, K, int(hidden.stride(0)), _ptr(weight), V,
+          int(weight.stride(0)), _ptr(out), _ptr(out_max), _ptr(workspace),
+          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
     return (out, out_max) if want_max or out_max is not None else out
 
 
@@ -417,10 +460,9 @@ def visual_importance(attn: torch.Tensor, v0: int, n_vis: int, r: int, workspace
     need = int(_lib().dreams_visual_importance_workspace_size(B, H, Q, n_vis))
     if workspace is None:
         workspace = _workspace("importance", need, dev, stream)
-    st = _lib().dreams_visual_importance(_ptr(attn), F32 if attn.dtype == torch.float32 else BF16, B, H, Q, K, v0,
-                                         n_vis, r, _ptr(imp), _ptr(keep), _ptr(workspace),
-                                         0 if workspace is None else workspace.numel(), _stream(stream))
-    _check("dreams_visual_importance", st)
+    _call("dreams_visual_importance", dev, _ptr(attn), F32 if attn.dtype == torch.float32 else BF16, B, H, Q, K, v0,
+          n_vis, r, _ptr(imp), _ptr(keep), _ptr(workspace), 0 if workspace is None else workspace.numel(),
+          _stream(stream, dev))
     return imp, keep
 
 
@@ -437,9 +479,8 @@ def accept_path(argmax: torch.Tensor, tree: Tree, max_path: int, status: Optiona
     dev = tree.parent.device
     _need(argmax, "argmax", torch.int32, dev)
     acc, path, toks, nkl = _walk_outputs(tree.B, max_path, dev)
-    st = _lib().dreams_accept_path(_ptr(argmax), ctypes.byref(tree._c), max_path, _ptr(acc), _ptr(path),
-                                   _ptr(toks), _ptr(nkl), _ptr(status), _stream(stream))
-    _check("dreams_accept_path", st)
+    _call("dreams_accept_path", dev, _ptr(argmax), ctypes.byref(tree._c), max_path, _ptr(acc), _ptr(path),
+          _ptr(toks), _ptr(nkl), _ptr(status), _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
 
@@ -450,9 +491,8 @@ def kv_compact(kv: KVCache, kv_len: torch.Tensor, accept_len: torch.Tensor, path
     for n, t in (("kv_len", kv_len), ("accept_len", accept_len), ("path", path)):
         _need(t, n, torch.int32, dev)
     B, max_path = (int(x) for x in path.shape)
-    st = _lib().dreams_kv_compact(ctypes.byref(kv._c), B, _ptr(kv_len), _ptr(accept_len), _ptr(path), max_path,
-                                  _ptr(status), _stream(stream))
-    _check("dreams_kv_compact", st)
+    _call("dreams_kv_compact", dev, ctypes.byref(kv._c), B, _ptr(kv_len), _ptr(accept_len), _ptr(path), max_path,
+          _ptr(status), _stream(stream, dev))
 
 
 def verify_step_sampled_workspace_size(tree: Tree, V: int) -> int:
@@ -482,12 +522,11 @@ def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
     need = verify_step_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step", need, dev, stream)
-    st = _lib().dreams_verify_step(
-        _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
-        ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, _ptr(argmax_out), _ptr(acc), _ptr(path),
-        _ptr(toks), _ptr(nkl), _ptr(workspace), 0 if workspace is None else workspace.numel(), _ptr(status),
-        _stream(stream))
-    _check("dreams_verify_step", st)
+    _call("dreams_verify_step", dev,
+          _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
+          ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, _ptr(argmax_out), _ptr(acc), _ptr(path),
+          _ptr(toks), _ptr(nkl), _ptr(workspace), 0 if workspace is None else workspace.numel(), _ptr(status),
+          _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
 
@@ -514,10 +553,17 @@ def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path:
     need = verify_step_sampled_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step_sampled", need, dev, stream)
-    st = _lib().dreams_verify_step_sampled(
-        _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
-        ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature), _ptr(uniforms),
-        _ptr(sample_out), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(workspace),
-        0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream))
-    _check("dreams_verify_step_sampled", st)
+    _call("dreams_verify_step_sampled", dev,
+          _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
+          ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature), _ptr(uniforms),
+          _ptr(sample_out), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(workspace),
+          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
+
+
+def test_set_stall(kernels: int, stall_at: int, wait_limit_ns: int = 20_000_000) -> None:
+    """Test hook for the bounded pipeline waits (``dreams_test_set_stall``):
+    later launches of the selected kernel families withhold their copies from
+    the ``stall_at``-th tile on and give up waiting after ``wait_limit_ns``.
+    ``stall_at < 0`` restores normal operation."""
+    _check("dreams_test_set_stall", _lib().dreams_test_set_stall(int(kernels), int(stall_at), int(wait_limit_ns)))

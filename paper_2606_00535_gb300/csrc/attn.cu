@@ -112,6 +112,8 @@ struct AttnParams {
   int32_t mode;    // ATTN_TREE, ATTN_FULL or ATTN_CAUSAL: which slots a query row attends
   float *ent;      // [B, T_max, Hq] attention entropy of each query row (nats), with the entropy kernels
   float *ws_w;     // [B][Hkv][nrb][nsplit][ROWS] sum_j P_j (x_j - m) of the split partials (entropy)
+  uint64_t wait_ns;  // limit of every pipeline wait (2 s unless a test shortens it)
+  int32_t stall_at;  // test hook: K tiles from this index on are never issued (-1: off)
 };
 
 constexpr int ATTN_TREE = 0;    // prefix slots plus the node's own ancestors among the tree slots
@@ -248,7 +250,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t bar_kf[NK], bar_ke[NK], bar_vf[NV], bar_ve[NV];
-  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_q, bar_drain;
+  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_q, bar_drain, bar_never;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_zero, s_flag;
   __shared__ unsigned long long s_anc[64];
@@ -317,7 +319,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const uint32_t kf0 = smem_u32(&bar_kf[0]), ke0 = smem_u32(&bar_ke[0]);
   const uint32_t vf0 = smem_u32(&bar_vf[0]), ve0 = smem_u32(&bar_ve[0]);
   const uint32_t bs0 = smem_u32(&bar_s[0]), bp0 = smem_u32(&bar_p[0]);
-  const uint32_t bq = smem_u32(&bar_q), bdrain = smem_u32(&bar_drain);
+  const uint32_t bq = smem_u32(&bar_q), bdrain = smem_u32(&bar_drain), bnever = smem_u32(&bar_never);
   const int t0 = rb * p.TB;  // first tree node of the row block
   const int c0 = split * p.chunk;
 
@@ -326,7 +328,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   // arrive: the producer sets up the copy barriers and issues both at once.
   // A CTA that then turns out to have nothing to do waits for them to land
   // before it exits.
-  const bool early = !P.paged && p.order == nullptr && !p.rank;
+  const bool early = !P.paged && p.order == nullptr && !p.rank && p.stall_at < 0;
   auto init_copy_barriers = [&]() {
     for (int i = 0; i < NK; ++i) {
       tc::mbar_init(kf0 + 8 * i, 1);
@@ -399,6 +401,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       tc::mbar_init(bp0 + 8 * i, 32 * n_act);
     }
     tc::mbar_init(bdrain, 1);
+    tc::mbar_init(bnever, 1);  // nothing arrives on it (the stall test hook waits on it)
     s_abort = 0;
     s_flag = 0;
     tc::fence_barrier_init();
@@ -415,6 +418,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const int c1 = ::min(c0 + p.chunk, kend);
   const int ntiles = (c1 - c0 + KT - 1) / KT;
   volatile int *abort_flag = &s_abort;
+  const uint64_t wait_ns = p.wait_ns;
   // abort codes: 1 = a wait timed out, 2 = malformed tree (nothing to compute)
   auto give_up = [&]() {
     if (*abort_flag == 0) {
@@ -521,6 +525,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         bool progress = false;
         if (nk < ntiles && nk - nv < CRD &&
             (nk < NK || tc::mbar_test_wait(ke0 + 8 * (nk % NK), ((nk / NK) - 1) & 1))) {
+          if (p.stall_at >= 0 && nk >= p.stall_at) {
+            // test hook: this copy is never issued; its consumers' waits run
+            // out, like this one on a barrier that nothing arrives on
+            tc::mbar_wait(bnever, 0, abort_flag, wait_ns);
+            give_up();
+            break;
+          }
           const int c3a = page_coord(nk, 0, pn0), c3b = page_coord(nk, 1, pn1);
           ring[nk % CRD][0] = c3a;
           ring[nk % CRD][1] = c3b;
@@ -557,7 +568,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           const uint64_t now = tc::global_ns();
           if (idle == 256u) {
             t_idle = now;
-          } else if (now - t_idle > 2000000000ull) {
+          } else if (now - t_idle > wait_ns) {
             give_up();
             break;
           }
@@ -603,8 +614,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           tc::mma_ts(tmem + ocol, tmem + scol + ks * 8, bd, IDESC_PV, (ii > 0 || ks > 0) ? 1u : 0u);
         }
       };
-      auto kwait = [&](int j) { return tc::mbar_wait(kf0 + 8 * (j % NK), (j / NK) & 1, abort_flag); };
-      bool ok = tc::mbar_wait(bq, 0, abort_flag) && kwait(0);
+      auto kwait = [&](int j) { return tc::mbar_wait(kf0 + 8 * (j % NK), (j / NK) & 1, abort_flag, wait_ns); };
+      bool ok = tc::mbar_wait(bq, 0, abort_flag, wait_ns) && kwait(0);
       if (ok) {
         tc::fence_after_sync();
         qk(0);
@@ -625,7 +636,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         const int w = j & 1;
         // P_j: the softmax warps arrive once one of them has also seen V_j
         // and K_{j+2} land
-        ok = tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag);
+        ok = tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag, wait_ns);
         if (!ok) break;
         tc::fence_after_sync();
         pv(j);
@@ -649,7 +660,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     bool ok = true;
     for (int ii = 0; ii < nw; ++ii) {
       const int j = 2 * ii + wg;
-      if (!__all_sync(0xffffffffu, tc::mbar_wait(bs0 + 8 * wg, ii & 1, abort_flag))) {
+      if (!__all_sync(0xffffffffu, tc::mbar_wait(bs0 + 8 * wg, ii & 1, abort_flag, wait_ns))) {
         give_up();
         ok = false;
         break;
@@ -751,7 +762,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         // PV product): zero those V rows before the MMA reads them, once the
         // tile's copy has landed (a later landing would undo the zeros)
         const int st = j % NV;
-        if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag))) {
+        if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag, wait_ns))) {
           give_up();
           ok = false;
           break;
@@ -780,8 +791,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       // stores): the MMA thread then waits for P_j alone.
       bool kv_ok = true;
       if (warp == 4 * wg && lane == 0)
-        kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag) &&
-                (j + 2 >= ntiles || tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag));
+        kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag, wait_ns) &&
+                (j + 2 >= ntiles ||
+                 tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag, wait_ns));
       if (!__all_sync(0xffffffffu, kv_ok)) {
         give_up();
         ok = false;
@@ -792,7 +804,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       tc::mbar_arrive(bp0 + 8 * wg);
     }
     // all MMAs done (the issuer commits this single-use barrier after its last PV)
-    if (ok && nw > 0 && !__all_sync(0xffffffffu, tc::mbar_wait(bdrain, 0, abort_flag))) {
+    if (ok && nw > 0 && !__all_sync(0xffffffffu, tc::mbar_wait(bdrain, 0, abort_flag, wait_ns))) {
       give_up();
       ok = false;
     }
@@ -870,6 +882,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           if (ENT) p.ws_w[slot + row] = Ls > 0.f ? Wt : 0.f;
         }
       }
+    } else if (act && *abort_flag == 1 && !direct && wg == 0 && real_row) {
+      // a wait gave up: the negative sum tells the merge to leave the row alone
+      p.ws_ml[slot + row] = make_float2(-INFINITY, -1.f);
     }
   }
 
@@ -934,6 +949,8 @@ __global__ void __launch_bounds__(256) tree_attn_merge_kernel(const AttnParams p
       bad |= (i == 0) ? (par != -1) : (par < 0 || par >= i);
     }
   }
+  // a split that gave up waiting left a negative sum: the row stays untouched
+  bad |= ml.y < 0.f;
   if (__any_sync(0xffffffffu, bad)) return;
 
   float M = ml.y > 0.f ? ml.x : -INFINITY;
@@ -1070,14 +1087,16 @@ bool make_kv_map(CUtensorMap *m, const void *base, const dreams_kv_cache_t *kv, 
 
 // 5-D view of the queries, (D, G, Hkv, T_max, B), with a (64 columns, G
 // heads, 1 KV head, TB nodes, 1) box: the query rows of one row block in
-// (node, head) order, 128-byte swizzle.
-bool make_q_map(CUtensorMap *m, const void *q, int B, int T_max, int Hq, int Hkv, int D, int TB) {
+// (node, head) order, 128-byte swizzle. A token's Hq head rows are dense;
+// tokens and sequences are q_stride_t and q_stride_b elements apart.
+bool make_q_map(CUtensorMap *m, const void *q, int B, int T_max, int Hq, int Hkv, int D, int TB, int64_t q_stride_b,
+                int64_t q_stride_t) {
   EncodeTiledFn enc = encode_tiled();
   if (enc == nullptr) return false;
   const int G = Hq / Hkv;
   const cuuint64_t dims[5] = {cuuint64_t(D), cuuint64_t(G), cuuint64_t(Hkv), cuuint64_t(T_max), cuuint64_t(B)};
-  const cuuint64_t strides[4] = {cuuint64_t(D) * 2, cuuint64_t(G) * D * 2, cuuint64_t(Hq) * D * 2,
-                                 cuuint64_t(T_max) * Hq * D * 2};
+  const cuuint64_t strides[4] = {cuuint64_t(D) * 2, cuuint64_t(G) * D * 2, cuuint64_t(q_stride_t) * 2,
+                                 cuuint64_t(q_stride_b) * 2};
   const cuuint32_t box[5] = {64, cuuint32_t(G), 1, cuuint32_t(TB), 1};
   const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(q), dims, strides, box, estr,
@@ -1109,26 +1128,19 @@ cudaError_t launch_pdl(const void *func, dim3 grid, dim3 block, size_t smem, cud
 
 template <int D, bool ENT>
 dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_cache_t *kv, const void *k,
-                       const void *v, int B, cudaStream_t stream) {
+                       const void *v, int B, int64_t q_stride_b, int64_t q_stride_t, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<D>();
-  static int configured_mask = 0;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 31 && !(configured_mask & (1 << dev))) {
-    cudaError_t e =
-        cudaFuncSetAttribute(tree_attn_tc_kernel<D, ENT>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-    if (e != cudaSuccess) {
-      set_last_cuda_error(e);
-      return DREAMS_ERR_CUDA;
-    }
-    configured_mask |= (1 << dev);
+  {
+    const dreams_status_t st =
+        ensure_max_dynamic_smem(reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT>), int(smem));
+    if (st != DREAMS_OK) return st;
   }
   TcParams P;
   memset(&P, 0, sizeof(P));
   P.a = a;
   P.paged = kv->page_table != nullptr;
   if (!make_kv_map(&P.tmap_k, k, kv, B) || !make_kv_map(&P.tmap_v, v, kv, B) ||
-      !make_q_map(&P.tmap_q, a.q, B, a.T_max, a.Hq, a.Hkv, D, a.TB))
+      !make_q_map(&P.tmap_q, a.q, B, a.T_max, a.Hq, a.Hkv, D, a.TB, q_stride_b, q_stride_t))
     return DREAMS_ERR_UNSUPPORTED;
   if (pl.ordered) {
     tree_attn_order_kernel<<<1, ORDER_THREADS, 0, stream>>>(a);
@@ -1165,7 +1177,8 @@ using namespace dreams;
 namespace {
 
 // The shared body of the two attention entry points.
-dreams_status_t attention_impl(const void *q, const dreams_kv_cache_t *kv, int32_t layer, const int32_t *parent,
+dreams_status_t attention_impl(const void *q, int64_t q_stride_b, int64_t q_stride_t, const dreams_kv_cache_t *kv,
+                               int32_t layer, const int32_t *parent,
                                const int32_t *q_len, const int32_t *kv_len, int32_t B, int32_t T_max, int32_t Hq,
                                float scale, int32_t mode, void *out, float *lse, float *ent, void *workspace,
                                size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream) {
@@ -1180,6 +1193,13 @@ dreams_status_t attention_impl(const void *q, const dreams_kv_cache_t *kv, int32
       (ent != nullptr && (reinterpret_cast<uintptr_t>(ent) & 3)))
     return DREAMS_ERR_INVALID_ARG;
   if (!isfinite(scale) || !(scale > 0.f)) return DREAMS_ERR_INVALID_ARG;
+  // Q rows: a token's head rows are dense, tokens and sequences are strided
+  // (16-byte multiples, as the tensor-map copy requires); with one sequence
+  // the sequence stride is not used
+  if (B == 1) q_stride_b = int64_t(T_max) * q_stride_t;
+  if (q_stride_t < int64_t(Hq) * kv->D || q_stride_b < int64_t(Hq) * kv->D || q_stride_t % 8 != 0 ||
+      q_stride_b % 8 != 0 || q_stride_t >= (int64_t(1) << 38) || q_stride_b >= (int64_t(1) << 38))
+    return DREAMS_ERR_INVALID_ARG;
   if (kv->page_table != nullptr) {
     if (kv->page_size != 64) return DREAMS_ERR_UNSUPPORTED;
     if (kv->pages_per_seq < 1 || kv->num_pages < 1 || int64_t(kv->pages_per_seq) * 64 != kv->capacity)
@@ -1225,12 +1245,15 @@ dreams_status_t attention_impl(const void *q, const dreams_kv_cache_t *kv, int32
   if (pl.ordered) p.order = reinterpret_cast<int32_t *>(ws + pl.ws_o_bytes + pl.ws_ml_bytes + pl.ws_w_bytes);
   p.rank = pl.ranked ? 1 : 0;
   p.status = status_word;
+  test_stall(DREAMS_TEST_ATTENTION, &p.stall_at, &p.wait_ns);
   const void *k = static_cast<const __nv_bfloat16 *>(kv->k) + int64_t(layer) * kv->layer_stride;
   const void *v = static_cast<const __nv_bfloat16 *>(kv->v) + int64_t(layer) * kv->layer_stride;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int64_t sb = q_stride_b, st = q_stride_t;
   if (want_ent)
-    return kv->D == 128 ? launch<128, true>(p, pl, kv, k, v, B, s) : launch<64, true>(p, pl, kv, k, v, B, s);
-  return kv->D == 128 ? launch<128, false>(p, pl, kv, k, v, B, s) : launch<64, false>(p, pl, kv, k, v, B, s);
+    return kv->D == 128 ? launch<128, true>(p, pl, kv, k, v, B, sb, st, s) : launch<64, true>(p, pl, kv, k, v, B, sb, st, s);
+  return kv->D == 128 ? launch<128, false>(p, pl, kv, k, v, B, sb, st, s)
+                      : launch<64, false>(p, pl, kv, k, v, B, sb, st, s);
 }
 
 }  // namespace
@@ -1249,13 +1272,14 @@ extern "C" int32_t dreams_tree_verify_attn_launches(const dreams_kv_cache_t *kv,
   return 1 + (pl.ordered ? 1 : 0) + (pl.nsplit > 1 ? 1 : 0);
 }
 
-extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+extern "C" dreams_status_t dreams_tree_verify_attn(const void *q, int64_t q_stride_b, int64_t q_stride_t,
+                                                   const dreams_kv_cache_t *kv, int32_t layer,
                                                    const dreams_tree_t *tree, int32_t Hq, float scale,
                                                    void *out, float *lse, void *workspace,
                                                    size_t workspace_bytes, int32_t *status_word,
                                                    dreams_stream_t stream) {
   if (tree == nullptr) return DREAMS_ERR_INVALID_ARG;
-  return attention_impl(q, kv, layer, tree->parent, tree->tree_len, tree->kv_len, tree->B, tree->T_max, Hq, scale,
+  return attention_impl(q, q_stride_b, q_stride_t, kv, layer, tree->parent, tree->tree_len, tree->kv_len, tree->B, tree->T_max, Hq, scale,
                         ATTN_TREE, out, lse, nullptr, workspace, workspace_bytes, status_word, stream);
 }
 
@@ -1265,12 +1289,13 @@ extern "C" size_t dreams_attention_workspace_size(const dreams_kv_cache_t *kv, i
   return plan(kv, B, T_max, Hq, want_entropy != 0).ws_bytes;
 }
 
-extern "C" dreams_status_t dreams_attention(const void *q, const dreams_kv_cache_t *kv, int32_t layer,
+extern "C" dreams_status_t dreams_attention(const void *q, int64_t q_stride_b, int64_t q_stride_t,
+                                            const dreams_kv_cache_t *kv, int32_t layer,
                                             const int32_t *q_len, const int32_t *kv_len, int32_t B, int32_t T_max,
                                             int32_t Hq, float scale, int32_t mode, void *out, float *lse,
                                             float *entropy, void *workspace, size_t workspace_bytes,
                                             int32_t *status_word, dreams_stream_t stream) {
   if (mode != DREAMS_ATTN_FULL && mode != DREAMS_ATTN_CAUSAL) return DREAMS_ERR_INVALID_ARG;
-  return attention_impl(q, kv, layer, nullptr, q_len, kv_len, B, T_max, Hq, scale, mode, out, lse, entropy,
+  return attention_impl(q, q_stride_b, q_stride_t, kv, layer, nullptr, q_len, kv_len, B, T_max, Hq, scale, mode, out, lse, entropy,
                         workspace, workspace_bytes, status_word, stream);
 }

@@ -16,6 +16,15 @@ void set_last_cuda_error(cudaError_t e);
 // Streaming multiprocessors of the current device (cached per device).
 int num_sms();
 
+// Sets a kernel's maximum dynamic shared memory on the current device, once
+// per (kernel, device); safe to call from several host threads.
+dreams_status_t ensure_max_dynamic_smem(const void *func, int bytes);
+
+// The stall test hook (dreams_test_set_stall) as it applies to one kernel
+// family: the index of the first withheld copy (-1: none) and the limit of
+// every pipeline wait (2 s unless the hook shortens it).
+void test_stall(int32_t kernel, int32_t *stall_at, uint64_t *wait_ns);
+
 inline dreams_status_t check_launch() {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {

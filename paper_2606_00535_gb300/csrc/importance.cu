@@ -380,18 +380,8 @@ extern "C" dreams_status_t dreams_visual_importance(const void *attn, dreams_dty
     if (st != DREAMS_OK) return st;
   }
   const size_t smem = size_t(n_vis) * 4;
-  static int configured_mask = 0;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 31 && !(configured_mask & (1 << dev))) {
-    const cudaError_t e = cudaFuncSetAttribute(importance_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               48 * 1024 * 4);
-    if (e != cudaSuccess) {
-      set_last_cuda_error(e);
-      return DREAMS_ERR_CUDA;
-    }
-    configured_mask |= (1 << dev);
-  }
+  st = ensure_max_dynamic_smem(reinterpret_cast<const void *>(importance_select_kernel), 48 * 1024 * 4);
+  if (st != DREAMS_OK) return st;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(unsigned(B));
   cfg.blockDim = dim3(SEL_THREADS);

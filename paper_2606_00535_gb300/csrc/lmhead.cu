@@ -19,7 +19,8 @@
 // CTAs working at one time share weight tiles through L2. A second kernel,
 // chained by programmatic dependent launch, turns each slot into the index
 // (and the maximum value) and resets it. Every wait is bounded (2 s); on a
-// timeout the CTA flags DREAMS_DATA_TIMEOUT in the status word, drains and
+// timeout the CTA flags DREAMS_DATA_TIMEOUT in the status word, merges no
+// further tile, waits for the copies and MMAs it issued, frees its TMEM and
 // exits.
 #include <cuda.h>
 #include <limits.h>
@@ -47,6 +48,8 @@ struct LmParams {
   int32_t nm, nn, nk;  // tiles along rows and vocabulary; k-blocks
   unsigned long long *slot;
   int32_t *status;
+  uint64_t wait_ns;  // limit of every pipeline wait (2 s unless a test shortens it)
+  int32_t stall_at;  // test hook: k-blocks from this index on (counted per CTA) are never issued (-1: off)
 };
 
 template <int dummy = 0>
@@ -54,7 +57,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
   constexpr uint32_t IDESC = tc::idesc_bf16_f32(BM, BN, false);
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_tf[2], bar_te[2];
+  __shared__ __align__(8) uint64_t bar_full[STAGES], bar_empty[STAGES], bar_tf[2], bar_te[2], bar_never;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_zero;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -72,6 +75,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
       tc::mbar_init(tf0 + 8 * i, 1);
       tc::mbar_init(te0 + 8 * i, 4);  // one arrival per epilogue warp
     }
+    tc::mbar_init(smem_u32(&bar_never), 1);  // nothing arrives on it (the stall test hook waits on it)
     s_abort = 0;
     s_zero = 0;
     tc::fence_barrier_init();
@@ -85,6 +89,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
   tc::fence_after_sync();
   const uint32_t tmem = s_tmem;
   volatile int *abort_flag = &s_abort;
+  const uint64_t wait_ns = P.wait_ns;
   auto give_up = [&]() {
     if (*abort_flag == 0) {
       *abort_flag = 1;
@@ -104,7 +109,14 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
         const int m = int(t % P.nm), n = int(t / P.nm);
         for (int kb = 0; kb < nk; ++kb, ++g) {
           const int st = int(g % STAGES);
-          if (g >= STAGES && !tc::mbar_wait(empty0 + 8 * st, ((g / STAGES) - 1) & 1, abort_flag)) {
+          if (g >= STAGES && !tc::mbar_wait(empty0 + 8 * st, ((g / STAGES) - 1) & 1, abort_flag, wait_ns)) {
+            give_up();
+            break;
+          }
+          if (P.stall_at >= 0 && g >= P.stall_at) {
+            // test hook: this copy is never issued; its consumers' waits run
+            // out, like this one on a barrier that nothing arrives on
+            tc::mbar_wait(smem_u32(&bar_never), 0, abort_flag, wait_ns);
             give_up();
             break;
           }
@@ -129,14 +141,14 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
       for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++it) {
         const int ab = it & 1;
         // the epilogue has read this accumulator's previous tile
-        if (it >= 2 && !tc::mbar_wait(te0 + 8 * ab, ((it >> 1) - 1) & 1, abort_flag)) {
+        if (it >= 2 && !tc::mbar_wait(te0 + 8 * ab, ((it >> 1) - 1) & 1, abort_flag, wait_ns)) {
           give_up();
           break;
         }
         tc::fence_after_sync();
         for (int kb = 0; kb < nk; ++kb, ++g) {
           const int st = int(g % STAGES);
-          if (!tc::mbar_wait(full0 + 8 * st, (g / STAGES) & 1, abort_flag)) {
+          if (!tc::mbar_wait(full0 + 8 * st, (g / STAGES) & 1, abort_flag, wait_ns)) {
             give_up();
             ok = false;
             break;
@@ -164,10 +176,13 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
     for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
       const int ab = it & 1;
       const int m = int(t % P.nm), n = int(t / P.nm);
-      if (!__all_sync(0xffffffffu, tc::mbar_wait(tf0 + 8 * ab, (it >> 1) & 1, abort_flag))) {
+      if (!__all_sync(0xffffffffu, tc::mbar_wait(tf0 + 8 * ab, (it >> 1) & 1, abort_flag, wait_ns))) {
         give_up();
         break;
       }
+      // after a give-up the MMA thread commits what it issued, so this
+      // accumulator may be unfinished: nothing more is merged
+      if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
       tc::fence_after_sync();
       const uint32_t taddr = tmem + (uint32_t(32 * q) << 16) + 256u * ab;
       const int64_t v0 = int64_t(n) * BN;
@@ -217,13 +232,16 @@ __global__ void __launch_bounds__(LM_THREADS, 1) lm_head_argmax_kernel(const __g
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// The row's index (and its maximum value) from its slot; resets the slot.
+// The row's index (and its maximum value) from its slot; resets the slot. A
+// slot that no tile reached (only when a wait gave up: every tile merges a
+// candidate, and no (key, index) pair packs to 0) leaves the row untouched.
 __global__ void __launch_bounds__(256) lm_head_finish_kernel(unsigned long long *slot, int64_t rows, int32_t *out_idx,
                                                              float *out_max) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t r = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (r >= rows) return;
   const unsigned long long v = slot[r];
+  if (v == 0ull) return;
   slot[r] = 0ull;
   out_idx[r] = int32_t(~uint32_t(v & 0xffffffffull));
   if (out_max != nullptr) {
@@ -288,17 +306,11 @@ extern "C" dreams_status_t dreams_lm_head_argmax(const void *hidden, int64_t row
   P.nk = int32_t(hidden_dim / BK);
   P.slot = static_cast<unsigned long long *>(workspace);
   P.status = status_word;
-  static int configured_mask = 0;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 31 && !(configured_mask & (1 << dev))) {
-    const cudaError_t e =
-        cudaFuncSetAttribute(lm_head_argmax_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(LM_SMEM));
-    if (e != cudaSuccess) {
-      set_last_cuda_error(e);
-      return DREAMS_ERR_CUDA;
-    }
-    configured_mask |= (1 << dev);
+  test_stall(DREAMS_TEST_LM_HEAD, &P.stall_at, &P.wait_ns);
+  {
+    const dreams_status_t st =
+        ensure_max_dynamic_smem(reinterpret_cast<const void *>(lm_head_argmax_kernel<0>), int(LM_SMEM));
+    if (st != DREAMS_OK) return st;
   }
   const int64_t ntiles = int64_t(P.nm) * P.nn;
   const unsigned grid = unsigned(std::min<int64_t>(ntiles, num_sms()));

@@ -105,13 +105,23 @@ def test_invalid_arguments_rejected_before_launch(lib):
     st = ctypes.c_void_p(P)
     s = ctypes.c_void_p(0)
 
-    def attn(q=P, kv=kvc, layer=0, tree=tr, Hq=4, scale=0.1, out=P, ws=None, wsb=0):
-        return lib.dreams_tree_verify_attn(q, ctypes.byref(kv), layer, ctypes.byref(tree), Hq, scale, out, null,
-                                           ws, wsb, st, s)
+    def attn(q=P, kv=kvc, layer=0, tree=tr, Hq=4, scale=0.1, out=P, ws=None, wsb=0, sb=8 * 4 * 128,
+             stt=4 * 128):
+        return lib.dreams_tree_verify_attn(q, sb, stt, ctypes.byref(kv), layer, ctypes.byref(tree), Hq, scale, out,
+                                           null, ws, wsb, st, s)
 
     assert attn(q=null) == dreams.ERR_INVALID_ARG
     assert attn(out=null) == dreams.ERR_INVALID_ARG
     assert attn(q=P + 2) == dreams.ERR_INVALID_ARG           # misaligned
+    # Q strides (elements): a fused-QKV view [B, T, 3, Hq, D] is accepted by
+    # the host checks; a token stride that is not a 16-byte multiple, one
+    # below the token's Hq * D head rows, or a short sequence stride is not
+    assert attn(stt=3 * 4 * 128 + 4) == dreams.ERR_INVALID_ARG
+    assert attn(stt=4 * 128 - 8) == dreams.ERR_INVALID_ARG
+    assert attn(sb=8 * 4 * 128 + 12) == dreams.ERR_INVALID_ARG
+    assert attn(sb=0) == dreams.ERR_INVALID_ARG
+    assert attn(stt=1 << 38) == dreams.ERR_INVALID_ARG
+    assert attn(stt=3 * 4 * 128, sb=8 * 3 * 4 * 128, q=null) == dreams.ERR_INVALID_ARG  # strides fine, q null
     assert attn(Hq=3) == dreams.ERR_INVALID_ARG              # Hq % Hkv
     assert attn(Hq=258) == dreams.ERR_INVALID_ARG            # more than 128 query heads per KV head
     assert attn(layer=1) == dreams.ERR_INVALID_ARG
@@ -153,3 +163,39 @@ def test_invalid_arguments_rejected_before_launch(lib):
               s) == dreams.ERR_INVALID_ARG
     assert vs(P, 3, 1000, 1000, ctypes.byref(tr), ctypes.byref(kvc), 5, null, P, P, P, P, P, wsb, st,
               s) == dreams.ERR_UNSUPPORTED
+
+
+def test_stall_hook_argument_checks(lib):
+    """The test hook of the bounded waits: only the two kernel families, a
+    wait limit of 1 us .. 2 s; a negative stall restores normal operation
+    whatever the other arguments."""
+    assert lib.dreams_test_set_stall(0, 0, 10_000_000) == dreams.ERR_INVALID_ARG
+    assert lib.dreams_test_set_stall(4, 0, 10_000_000) == dreams.ERR_INVALID_ARG
+    assert lib.dreams_test_set_stall(dreams.TEST_ATTENTION, 0, 999) == dreams.ERR_INVALID_ARG
+    assert lib.dreams_test_set_stall(dreams.TEST_LM_HEAD, 0, 2_000_000_001) == dreams.ERR_INVALID_ARG
+    assert lib.dreams_test_set_stall(dreams.TEST_ATTENTION | dreams.TEST_LM_HEAD, 3, 10_000_000) == dreams.OK
+    assert lib.dreams_test_set_stall(7, -1, 0) == dreams.OK
+
+
+def test_binding_checks_before_any_call():
+    """The wrappers refuse on the host, before any library call: a no-allocation
+    argmax over more rows than its fixed scratch, an output shorter than the
+    rows written, leading dimensions that flatten only by copying (which would
+    allocate), and a query tensor whose head rows are not dense."""
+    x = torch.zeros((dreams.NOALLOC_ARGMAX_MAX_ROWS + 1, 8), dtype=torch.float32)
+    out = torch.zeros(dreams.NOALLOC_ARGMAX_MAX_ROWS + 1, dtype=torch.int32)
+    with pytest.raises(ValueError, match="fixed scratch"):
+        dreams.vocab_argmax_noalloc(x, out)
+    x = torch.zeros((6, 8), dtype=torch.float32)
+    with pytest.raises(ValueError, match="holds 5 elements"):
+        dreams.vocab_argmax_noalloc(x, torch.zeros(5, dtype=torch.int32))
+    with pytest.raises(ValueError, match="holds 5 elements"):
+        dreams.vocab_argmax(x, out=torch.zeros(5, dtype=torch.int32))
+    y = torch.zeros((4, 3, 8), dtype=torch.float32).transpose(0, 1)  # [3, 4, 8], not viewable as [12, 8]
+    with pytest.raises(ValueError, match="without a copy"):
+        dreams.vocab_argmax_noalloc(y, torch.zeros(12, dtype=torch.int32))
+    q = torch.zeros((2, 5, 4, 64), dtype=torch.bfloat16).transpose(2, 1)  # heads strided
+    with pytest.raises(ValueError, match="head rows must be dense"):
+        dreams._q_strides(q)
+    fused = torch.zeros((2, 5, 3, 4, 64), dtype=torch.bfloat16)
+    assert dreams._q_strides(fused[:, :, 0]) == (5 * 3 * 4 * 64, 3 * 4 * 64)
