@@ -27,11 +27,12 @@ def dreams():
     d.test_set_stall(0, -1)
 
 
-def _uneven_case(dreams):
+def _uneven_case(dreams, Hq):
     """Five sequences: two fit in one 128-key tile (they finish before any
-    stall at the second tile), three span 12 to 32 tiles."""
+    stall at the second tile), three span 12 to 32 tiles. With 4 query heads
+    per KV head the 24 nodes fill one row block per KV head; with 8, two."""
     rng = np.random.default_rng(77)
-    B, Hq, Hkv, D, T, cap = 5, 8, 2, 128, 24, 4096
+    B, Hkv, D, T, cap = 5, 2, 128, 24, 4096
     par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
     tl = np.array([24, 1, 17, 24, 9], np.int32)
     for b in range(B):
@@ -56,8 +57,9 @@ def _attend(dreams, q, kv, tree, scale):
     return out.view(torch.int16).clone(), lse.clone(), int(st.item())
 
 
-def test_attention_wait_runs_out_then_recovers(dreams):
-    q, kv, tree, tl, scale = _uneven_case(dreams)
+@pytest.mark.parametrize("Hq", [8, 16])
+def test_attention_wait_runs_out_then_recovers(dreams, Hq):
+    q, kv, tree, tl, scale = _uneven_case(dreams, Hq)
     ref_out, ref_lse, st = _attend(dreams, q, kv, tree, scale)
     assert st == 0
     try:
@@ -74,13 +76,14 @@ def test_attention_wait_runs_out_then_recovers(dreams):
     assert torch.equal(out2, ref_out) and torch.equal(lse2, ref_lse)
 
 
-def test_attention_partial_stall_leaves_unfinished_rows_untouched(dreams):
+@pytest.mark.parametrize("Hq", [8, 16])
+def test_attention_partial_stall_leaves_unfinished_rows_untouched(dreams, Hq):
     """Copies withheld from the second K tile on: the one-tile sequences (1 and
     3) finish and match the normal call bit for bit; every row of the long
     ones, whether written directly or through the merge of the KV splits (a
     KV split spans at least two tiles, so the first split of every row block
     gives up and tells the merge to skip the row), is untouched."""
-    q, kv, tree, tl, scale = _uneven_case(dreams)
+    q, kv, tree, tl, scale = _uneven_case(dreams, Hq)
     ref_out, ref_lse, _ = _attend(dreams, q, kv, tree, scale)
     try:
         dreams.test_set_stall(dreams.TEST_ATTENTION, 1, 20_000_000)
