@@ -262,9 +262,14 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   const int per_pair = p.Hkv * p.nrb;
   const int pair_pos = blockIdx.x / per_pair;
   const int gr = blockIdx.x - pair_pos * per_pair;
-  const int g = gr / p.nrb, rb_raw = gr - g * p.nrb;
-  // causal rows: the last row blocks have the most keys, so they go first
-  const int rb = p.mode == ATTN_CAUSAL ? p.nrb - 1 - rb_raw : rb_raw;
+  // Tree and cross-attention rows: KV head, then row block (the row blocks of
+  // a head, adjacent, share its K/V tiles through L2). Causal rows: the last
+  // row blocks have the most keys, so the order is row block (last first),
+  // then KV head: the hardware, handing out CTAs in index order, then
+  // schedules longest first.
+  const bool causal = p.mode == ATTN_CAUSAL;
+  const int g = causal ? gr % p.Hkv : gr / p.nrb;
+  const int rb = causal ? p.nrb - 1 - gr / p.Hkv : gr - g * p.nrb;
   int pair = pair_pos;
   if (p.order != nullptr) {
     // the order comes from the preceding kernel (programmatic dependent launch)
