@@ -32,6 +32,9 @@ paper passage its C routine follows:
   Target Feature Injection") or a layer's causal prefill (query t sees slots
   0 .. L+t), with each row's attention entropy -sum_j a_j ln a_j, whose mean
   over rows and heads is AE(l) (Sec. 3.3).
+* :func:`spec_path` -- speculative sampling over the tree (Leviathan et al.,
+  cited in Sec. 1; T = 1 in Table 2): drafts accepted with probability
+  min(1, p/q), the bonus drawn from the renormalised residual max(0, p - q).
 * :func:`accept_path` -- sequential acceptance with the target's token
   replacing the first mismatch (Sec. 2 "Speculative decoding"), over a tree.
 * :func:`kv_compact` -- the accepted nodes' K/V moved into contiguous slots
@@ -98,6 +101,10 @@ def _load() -> ctypes.CDLL:
         _lib.oracle_sample_bf16.restype = None
         _lib.oracle_accept_path.argtypes = [p, p, p, p, p, i64, i64, i64, p, p, p, p]
         _lib.oracle_accept_path.restype = ctypes.c_int
+        for nm in ("oracle_spec_path_f32", "oracle_spec_path_bf16"):
+            fn = getattr(_lib, nm)
+            fn.argtypes = [p, p, i64, i64, p, p, p, p, i64, i64, i64, f64, p, p, p, p, p, p, p]
+            fn.restype = ctypes.c_int
         _lib.oracle_kv_compact.argtypes = [
             p, p, i64, i64, i64, p, i64, i64, i64, i64, i64, i64, p, p, p, i64]
         _lib.oracle_kv_compact.restype = ctypes.c_int
@@ -296,6 +303,36 @@ def accept_path(am, parent, tokens, tree_len, kv_len, max_path: int):
     st = _load().oracle_accept_path(_ptr(am), _ptr(par), _ptr(tok), _ptr(tl), _ptr(kl), B, T_max,
                                     max_path, _ptr(acc), _ptr(path), _ptr(outt), _ptr(nkl))
     return {"accept_len": acc, "path": path, "out_tokens": outt, "new_kv_len": nkl, "status": st}
+
+
+def spec_path(target, draft, parent, tokens, tree_len, kv_len, max_path: int, temperature: float, u_accept,
+              u_resample, bf16_bits: bool = False):
+    """Speculative sampling over the draft trees (Leviathan et al., cited in
+    Sec. 1; verification at T = 1, Table 2) -- see ``oracle_spec_path`` in
+    oracle.c. target, draft: [B, T_max, V] logits (float32, or uint16 bf16
+    patterns); u_accept, u_resample: float32 [B, T_max]. Returns dict of
+    accept_len, path, out_tokens, new_kv_len, the OR of data-error bits and
+    margin [B] (the smallest distance of a uniform from its threshold)."""
+    par = _c(parent, np.int32)
+    B, T_max = par.shape
+    dt = np.uint16 if bf16_bits else np.float32
+    t = _c(target, dt)
+    d = _c(draft, dt)
+    V = t.shape[-1]
+    t = t.reshape(B * T_max, V)
+    d = d.reshape(B * T_max, V)
+    acc = np.empty((B,), np.int32)
+    path = np.empty((B, max_path), np.int32)
+    outt = np.empty((B, max_path), np.int32)
+    nkl = np.empty((B,), np.int32)
+    mg = np.empty((B,), np.float64)
+    fn = _load().oracle_spec_path_bf16 if bf16_bits else _load().oracle_spec_path_f32
+    st = fn(_ptr(t), _ptr(d), V, V, _ptr(par), _ptr(_c(tokens, np.int32)), _ptr(_c(tree_len, np.int32)),
+            _ptr(_c(kv_len, np.int32)), B, T_max, max_path, float(temperature),
+            _ptr(_c(np.asarray(u_accept, np.float32).reshape(B, T_max), np.float32)),
+            _ptr(_c(np.asarray(u_resample, np.float32).reshape(B, T_max), np.float32)),
+            _ptr(acc), _ptr(path), _ptr(outt), _ptr(nkl), _ptr(mg))
+    return {"accept_len": acc, "path": path, "out_tokens": outt, "new_kv_len": nkl, "status": st, "margin": mg}
 
 
 def kv_compact(k_bits, v_bits, layout: KVLayout, kv_len, accept_len, path, n_layers: int = 1,

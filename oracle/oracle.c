@@ -32,6 +32,12 @@
  *                             mismatch (Sec. 2 "Speculative decoding"),
  *                             generalised from a chain to the longest matching
  *                             root path of a draft tree.
+ *   - oracle_spec_path_*    : speculative sampling over the draft tree
+ *                             (Leviathan et al., cited in Sec. 1): each draft
+ *                             is accepted with probability min(1, p / q),
+ *                             and a rejection moves the target to the
+ *                             renormalised residual max(0, p - q) from which
+ *                             the bonus token is drawn (Table 2, T = 1).
  *   - oracle_kv_compact     : the accepted nodes' K/V are moved into the
  *                             contiguous slots that follow the prefix, so the
  *                             cache stays a plain sequence for the next step
@@ -411,6 +417,164 @@ int oracle_accept_path(const int32_t *am, const int32_t *parent, const int32_t *
   free(best);
   free(cand);
   return status;
+}
+
+/* Target or draft distribution of a row: w_v = exp((x_v - M) / tau) / Z. */
+static void row_softmax(const double *x, int64_t V, double tau, double *w) {
+  double M = -INFINITY;
+  for (int64_t v = 0; v < V; ++v)
+    if (x[v] > M) M = x[v];
+  double Z = 0.0;
+  for (int64_t v = 0; v < V; ++v) {
+    w[v] = exp((x[v] - M) / tau);
+    Z += w[v];
+  }
+  for (int64_t v = 0; v < V; ++v) w[v] /= Z;
+}
+
+/* Inverse-transform draw from a distribution w (sums to 1 up to rounding):
+ * the smallest v with w_0 + ... + w_v > u, u clamped to [0, 1] (NaN counts as
+ * 0); none (u = 1): the last v with w_v > 0. *margin gets min(its current
+ * value, the distance of u from the nearest cumulative sum). */
+static int64_t draw_dist(const double *w, int64_t V, double u, double *margin) {
+  if (!(u > 0.0)) u = 0.0;
+  if (u > 1.0) u = 1.0;
+  double cum = 0.0;
+  int64_t last = 0;
+  for (int64_t v = 0; v < V; ++v) {
+    const double before = cum;
+    cum += w[v];
+    if (w[v] > 0.0) last = v;
+    if (cum > u) {
+      const double d = fmin(u - before, cum - u);
+      if (d < *margin) *margin = d;
+      return v;
+    }
+  }
+  return last;
+}
+
+/*
+ * Speculative sampling over a draft tree (Leviathan et al., cited in Sec. 1;
+ * the verification at temperature 1 of Table 2), walked from the root: at
+ * node cur the target's distribution is p = softmax(target[cur] / tau) and
+ * the draft's is q = softmax(draft[cur] / tau), the distribution the drafts
+ * of cur's children were drawn from. The children are tried in index order,
+ * with the residual r = p at first: child c with draft token x is accepted
+ * when u_acc[c] < min(1, r(x) / q(x)) (q(x) = 0: accepted when r(x) > 0);
+ * a rejection replaces r by max(0, r - q) / sum max(0, r - q) (kept as it is
+ * when that sum is 0, i.e. r == q). An accepted child becomes cur. When no
+ * child is accepted, at a leaf, or once max_path - 1 drafts are accepted,
+ * the bonus token is drawn from r (p at a leaf or at the cut) by inverse
+ * transform with u_res[cur], and the walk stops. Outputs as
+ * oracle_accept_path: path, out_tokens (accepted drafts then the bonus),
+ * accept_len = n + 1, new_kv_len = kv_len + n + 1; a malformed tree or
+ * kv_len < 0 gets accept_len 0 and rows of -1. margin[b] (may be NULL): the
+ * smallest distance of a uniform from the threshold it was compared with
+ * (|u_acc - min(1, r/q)| per tested child, the distance to the nearest
+ * cumulative sum for the draw), so a test can tell which decisions a
+ * rounding difference could flip. target / draft: B * T_max rows of V values
+ * (row b * T_max + i is node i of sequence b), row_stride apart; the draft
+ * rows of leaves are not read.
+ */
+static int spec_path(const void *target, const void *draft, int bf16, int64_t V, int64_t row_stride,
+                     const int32_t *parent, const int32_t *tokens, const int32_t *tree_len, const int32_t *kv_len,
+                     int64_t B, int64_t T_max, int64_t max_path, double tau, const float *u_acc,
+                     const float *u_res, int32_t *accept_len, int32_t *path, int32_t *out_tokens,
+                     int32_t *new_kv_len, double *margin) {
+  int status = 0;
+  double *x = (double *)malloc((size_t)V * sizeof(double));
+  double *p = (double *)malloc((size_t)V * sizeof(double));
+  double *q = (double *)malloc((size_t)V * sizeof(double));
+  for (int64_t b = 0; b < B; ++b) {
+    const int32_t *par = parent + b * T_max;
+    const int32_t *tok = tokens + b * T_max;
+    int32_t *pb = path + b * max_path;
+    int32_t *ob = out_tokens + b * max_path;
+    double mg = INFINITY;
+    for (int64_t k = 0; k < max_path; ++k) pb[k] = ob[k] = -1;
+    int bad = check_tree(par, tree_len[b], (int32_t)T_max);
+    if (!bad && kv_len[b] < 0) bad = ORACLE_BAD_KV_LEN;
+    if (bad || max_path < 1) {
+      status |= bad;
+      accept_len[b] = 0;
+      new_kv_len[b] = kv_len[b];
+      if (margin) margin[b] = mg;
+      continue;
+    }
+    const int32_t T = tree_len[b];
+    int32_t cur = 0, n = 0;
+    pb[0] = 0;
+    for (;;) {
+      const int64_t row = b * T_max + cur;
+      for (int64_t v = 0; v < V; ++v)
+        x[v] = bf16 ? bf16_bits_to_double(((const uint16_t *)target)[row * row_stride + v])
+                    : (double)((const float *)target)[row * row_stride + v];
+      row_softmax(x, V, tau, p); /* p now holds the residual r, which starts as the target */
+      int32_t next = -1;
+      if (n < max_path - 1) {
+        int have_q = 0;
+        for (int32_t c = cur + 1; c < T && next < 0; ++c) {
+          if (par[c] != cur) continue;
+          if (!have_q) {
+            for (int64_t v = 0; v < V; ++v)
+              x[v] = bf16 ? bf16_bits_to_double(((const uint16_t *)draft)[row * row_stride + v])
+                          : (double)((const float *)draft)[row * row_stride + v];
+            row_softmax(x, V, tau, q);
+            have_q = 1;
+          }
+          const int32_t t = tok[c];
+          const double r_t = (t >= 0 && t < V) ? p[t] : 0.0;
+          const double q_t = (t >= 0 && t < V) ? q[t] : 0.0;
+          const double a = q_t > 0.0 ? fmin(1.0, r_t / q_t) : (r_t > 0.0 ? 1.0 : 0.0);
+          const double u = (double)u_acc[b * T_max + c];
+          if (fabs(u - a) < mg) mg = fabs(u - a);
+          if (u < a) {
+            next = c;
+          } else {
+            double Z = 0.0;
+            for (int64_t v = 0; v < V; ++v) Z += fmax(0.0, p[v] - q[v]);
+            if (Z > 0.0)
+              for (int64_t v = 0; v < V; ++v) p[v] = fmax(0.0, p[v] - q[v]) / Z;
+          }
+        }
+      }
+      if (next < 0) {
+        const int64_t bonus = draw_dist(p, V, (double)u_res[b * T_max + cur], &mg);
+        ob[n] = (int32_t)bonus;
+        break;
+      }
+      ++n;
+      pb[n] = next;
+      ob[n - 1] = tok[next];
+      cur = next;
+    }
+    accept_len[b] = n + 1;
+    new_kv_len[b] = kv_len[b] + n + 1;
+    if (margin) margin[b] = mg;
+  }
+  free(x);
+  free(p);
+  free(q);
+  return status;
+}
+
+int oracle_spec_path_f32(const float *target, const float *draft, int64_t V, int64_t row_stride,
+                         const int32_t *parent, const int32_t *tokens, const int32_t *tree_len,
+                         const int32_t *kv_len, int64_t B, int64_t T_max, int64_t max_path, double tau,
+                         const float *u_acc, const float *u_res, int32_t *accept_len, int32_t *path,
+                         int32_t *out_tokens, int32_t *new_kv_len, double *margin) {
+  return spec_path(target, draft, 0, V, row_stride, parent, tokens, tree_len, kv_len, B, T_max, max_path, tau,
+                   u_acc, u_res, accept_len, path, out_tokens, new_kv_len, margin);
+}
+
+int oracle_spec_path_bf16(const uint16_t *target, const uint16_t *draft, int64_t V, int64_t row_stride,
+                          const int32_t *parent, const int32_t *tokens, const int32_t *tree_len,
+                          const int32_t *kv_len, int64_t B, int64_t T_max, int64_t max_path, double tau,
+                          const float *u_acc, const float *u_res, int32_t *accept_len, int32_t *path,
+                          int32_t *out_tokens, int32_t *new_kv_len, double *margin) {
+  return spec_path(target, draft, 1, V, row_stride, parent, tokens, tree_len, kv_len, B, T_max, max_path, tau,
+                   u_acc, u_res, accept_len, path, out_tokens, new_kv_len, margin);
 }
 
 /*
