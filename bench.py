@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sampled", action="store_true",
                     help="skip the extra timing of the temperature-1 verification tail")
+    ap.add_argument("--no-speculative", action="store_true",
+                    help="skip the extra timing of the speculative-sampling verification tail")
     ap.add_argument("--no-lm-head", action="store_true",
                     help="skip the extra timing of the LM head with the fused argmax")
     ap.add_argument("--no-modes", action="store_true",
@@ -88,6 +90,16 @@ def attn_bytes(w: W.Workload) -> int:
 def argmax_bytes(w: W.Workload) -> int:
     """Algorithmic bytes of the argmax: every logit of every tree node once."""
     return int(w.tree_len.sum()) * w.V * (4 if w.logits_dtype == "f32" else 2)
+
+
+def speculative_bytes(w: W.Workload) -> int:
+    """Algorithmic bytes of the speculative tail: the target row of every
+    tree node and the draft row of every node with children, each once."""
+    inner = 0
+    for b in range(w.B):
+        par = w.parent[b, :int(w.tree_len[b])].numpy()
+        inner += len(set(int(x) for x in par[1:]))
+    return argmax_bytes(w) + inner * w.V * (4 if w.logits_dtype == "f32" else 2)
 
 
 def attn_flops(w: W.Workload) -> int:
@@ -495,6 +507,46 @@ def run_dreams(args, rank, world, local):
         sampled = {"us": round(sampled_us, 2), "temperature": 1.0, "launches": dreams.VERIFY_STEP_SAMPLED_LAUNCHES,
                    "launch": "eager", "GBps": round(argmax_bytes(w) / (sampled_us * 1e-6) / 1e9, 1)}
 
+    # ---- speculative sampling over the tree at temperature 1: draft logits =
+    # target + N(0, 0.5) noise, drafts accepted with probability min(1, r/q)
+    speculative = None
+    if not args.no_speculative:
+        g = torch.Generator(device=dev).manual_seed(11)
+        drafts = [(c["logits"].float() + 0.5 * torch.randn(c["logits"].shape, generator=g, device=dev)).to(
+            c["logits"].dtype) for c in copies]
+        cpu_g = torch.Generator().manual_seed(13)
+        u_a = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
+        u_r = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
+        ws_sp = torch.zeros(dreams.verify_step_speculative_workspace_size(copies[0]["tree"], w.V),
+                            dtype=torch.uint8, device=dev)
+
+        def spec_call(i):
+            c = copies[i % 2]
+            dreams.verify_step_speculative(c["logits"], drafts[i % 2], c["tree"], c["kv"], max_path, 1.0, u_a, u_r,
+                                           outputs=c["outs"], workspace=ws_sp, status=status)
+
+        for i in range(4):
+            spec_call(i)
+        Ks = max(3, min(K, 100))
+        s0 = torch.cuda.Event(enable_timing=True)
+        s1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        s0.record(stream)
+        for i in range(Ks):
+            spec_call(i)
+        s1.record(stream)
+        barrier()
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item()):#x} on valid input (speculative step)")
+        acc_mean = float(copies[(Ks - 1) % 2]["outs"][0].float().mean())
+        spec_us = s0.elapsed_time(s1) / Ks * 1000.0
+        sb = speculative_bytes(w)
+        speculative = {"us": round(spec_us, 2), "temperature": 1.0,
+                       "launches": dreams.VERIFY_STEP_SPECULATIVE_LAUNCHES, "launch": "eager",
+                       "bytes": sb, "GBps": round(sb / (spec_us * 1e-6) / 1e9, 1),
+                       "draft": "target logits + N(0, 0.5) noise", "mean_accept_len": round(acc_mean, 3)}
+        del drafts
+
     # ---- the LM head with its argmax fused (the logits never reach HBM), on
     # the tree rows of this workload: hidden size Hq * D, random bf16 weights
     lm_head = None
@@ -658,6 +710,9 @@ def run_dreams(args, rank, world, local):
     if sampled is not None:
         sampled["frac_measured_hbm"] = round(sampled["GBps"] / peak, 4)
         kernels["verify_step_sampled"] = sampled
+    if speculative is not None:
+        speculative["frac_measured_hbm"] = round(speculative["GBps"] / peak, 4)
+        kernels["verify_step_speculative"] = speculative
     if lm_head is not None:
         kernels["lm_head_argmax"] = lm_head
     if importance is not None:

@@ -301,6 +301,48 @@ dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dt
                                            dreams_stream_t stream);
 
 /*
+ * The verification tail at temperature tau > 0 by speculative sampling
+ * (Leviathan et al., cited in Sec. 1; Table 2, Temperature = 1), over the
+ * draft tree: the accepted tokens are distributed as the target's own samples
+ * whatever the draft proposes. At node cur the target's distribution is
+ * p = softmax(target[cur] / tau) and the draft's q = softmax(draft[cur] / tau),
+ * the distribution the drafts of cur's children were drawn from. The walk
+ * starts at the root with the residual r = p and tries cur's children in index
+ * order: child c with draft token x is accepted when
+ *     u_accept[b][c] < min(1, r(x) / q(x))        (q(x) = 0: accepted iff r(x) > 0)
+ * and then becomes cur (r restarts as the target at c); a rejection replaces r
+ * by max(0, r - q) / sum_v max(0, r - q) (kept when that sum is 0, r == q).
+ * When no child is accepted, at a leaf, or once max_path - 1 drafts are
+ * accepted, the bonus token is drawn from r by inverse transform with
+ * u_resample[b][cur] (the smallest v whose cumulative weight exceeds u, u
+ * clamped to [0, 1]; none: the last v of positive weight). accept_len, path,
+ * out_tokens, new_kv_len and the KV compaction are as in dreams_verify_step.
+ * target_logits, draft_logits: f32 or bf16, [B, T_max, V] with row_stride
+ * (the same for both); the draft rows of leaves are not read. u_accept,
+ * u_resample: device f32 [B, T_max] (the caller's random numbers). Logits must
+ * be finite (with non-finite values the tokens drawn are unspecified but lie in
+ * [0, V)). V <= 524288, max_path <= 65. Arithmetic is f32 (hardware exp2 of the
+ * scaled differences), so a decision can differ from the exact-arithmetic one
+ * only when a uniform lies within rounding of its threshold. Two launches,
+ * chained by programmatic dependent launch: the 1024-value segment statistics
+ * of the target rows of the tree nodes and of the draft rows of nodes with
+ * children (8 bytes per 1024 values per row in the workspace); then one CTA
+ * per sequence that walks the tree, taking one pass over both rows of a node
+ * for each rejection there (the residual's sum), draws the bonus, writes the
+ * outputs and moves the accepted K/V. The workspace holds no state between
+ * calls.
+ */
+size_t dreams_verify_step_speculative_workspace_size(const dreams_tree_t *tree, int64_t V);
+dreams_status_t dreams_verify_step_speculative(const void *target_logits, const void *draft_logits,
+                                               dreams_dtype_t dtype, int64_t V, int64_t row_stride,
+                                               const dreams_tree_t *tree, const dreams_kv_cache_t *kv,
+                                               int32_t max_path, float temperature, const float *u_accept,
+                                               const float *u_resample, int32_t *accept_len, int32_t *path,
+                                               int32_t *out_tokens, int32_t *new_kv_len, void *workspace,
+                                               size_t workspace_bytes, int32_t *status_word,
+                                               dreams_stream_t stream);
+
+/*
  * The LM head with its argmax fused: the target's greedy prediction per node
  * straight from its final hidden states (Sec. 2 "Speculative decoding" at
  * temperature 0), without writing the logits:

@@ -1011,6 +1011,335 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
   if (n > 0) compact_units(p.kv, n, s_src, s_dst, threadIdx.x, blockDim.x);
 }
 
+// ------------------------------------------------------------------ speculative sampling
+// Verification at temperature tau by speculative sampling (Leviathan et al.,
+// cited in the paper's Sec. 1; T = 1 in Table 2), over the draft tree: at node
+// cur the target's distribution is p = softmax(target[cur] / tau) and the
+// draft's q = softmax(draft[cur] / tau), from which the drafts of cur's
+// children were drawn. Children are tried in index order against the residual
+// r (p at first): child c with draft x is accepted when u_acc[c] <
+// min(1, r(x) / q(x)); a rejection replaces r by max(0, r - q) / Z with
+// Z = sum max(0, r - q) (kept when Z = 0). The bonus is drawn from r by
+// inverse transform with u_res of the node where the walk stops.
+constexpr int SPEC_THREADS = 512;     // walk kernel: 16 warps share the passes over a row
+constexpr int SPEC_MAX_SEG = 512;     // 1024-value segments per row the walk keeps sums of (V <= 524288)
+
+struct SpecParams {
+  SampleParams tgt, drf;  // 1024-value segment statistics (m, sum 2^((x - m) k2)) of target and draft rows
+  TreeParams tr;
+  KVParams kv;
+  int32_t max_path;
+  const float *u_acc, *u_res;  // [B, T_max] each
+  int32_t *accept_len, *path, *out_tokens, *new_kv_len;
+  int32_t *status;
+};
+
+// Launch 1: statistics of the target rows of the tree nodes and of the draft
+// rows of nodes that have children. grid.x = 2 * B * T_max * ncta_row: (row
+// set, node row, CTA of the row); rows that are not needed return at once.
+template <typename T>
+__global__ void __launch_bounds__(SAMPLE_THREADS, sizeof(T) == 2 ? 6 : 4) spec_stats_kernel(const SpecParams p) {
+  const int ncta = p.tgt.ncta_row;
+  const int64_t rows = int64_t(p.tr.B) * p.tr.T_max;
+  const int64_t x = blockIdx.x / ncta;
+  const bool drf = x >= rows;
+  const int64_t r = drf ? x - rows : x;
+  const int b = int(r / p.tr.T_max), i = int(r % p.tr.T_max);
+  const int tl = __ldg(p.tr.tree_len + b);
+  bool live = tl >= 1 && tl <= p.tr.T_max && i < tl;
+  if (live && drf) {  // only a node with children has a draft distribution to read
+    bool kids = false;
+    for (int c = i + 1; c < tl && !kids; ++c) kids = __ldg(p.tr.parent + int64_t(b) * p.tr.T_max + c) == i;
+    live = kids;
+  }
+  if (live) {
+    const SampleParams &sp = drf ? p.drf : p.tgt;
+    const int64_t g0 = int64_t(blockIdx.x % ncta) * sp.seg_per_cta;
+    const int64_t g1 = std::min<int64_t>(sp.nseg, g0 + sp.seg_per_cta);
+    sample_stats<T>(sp, static_cast<const T *>(sp.logits) + r * sp.row_stride, sp.seg + r * sp.nseg, g0, g1);
+  }
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// (M, Z) of a row from its segment statistics, Z = sum_v 2^((x_v - M) k2); one
+// warp. The statistics were written by the preceding grid: read through L2.
+__device__ float2 spec_row_mz(const float2 *seg_row, int nseg, float k2) {
+  const int lane = threadIdx.x & 31;
+  float m_l = -INFINITY, z_l = 0.f;
+  for (int g = lane; g < nseg; g += 32) {
+    const float2 v = __ldcg(seg_row + g);
+    if (v.x == -INFINITY) continue;
+    if (v.x > m_l) {
+      z_l = (m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - v.x) * k2)) + v.y;
+      m_l = v.x;
+    } else {
+      z_l += v.y * exp2f_approx((v.x - m_l) * k2);
+    }
+  }
+  float M = m_l;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  float Z = m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - M) * k2);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Z += __shfl_xor_sync(0xffffffffu, Z, off);
+  return make_float2(M, Z);
+}
+
+// The residual after k rejections at a node, at one vocabulary entry, from
+// the target and draft probabilities there: r_0 = p, r_j = max(0, r_{j-1} - q) /
+// Z_j (kept when Z_j = 0).
+__device__ __forceinline__ float spec_residual(float pv, float qv, const float *zk, int k) {
+  float r = pv;
+  for (int j = 0; j < k; ++j) {
+    const float z = zk[j];
+    if (z > 0.f) r = fmaxf(r - qv, 0.f) / z;
+  }
+  return r;
+}
+
+// Launch 2, one CTA per sequence (chained to launch 1 by programmatic
+// dependent launch): the walk with its decisions, the bonus draw, the outputs
+// and the KV compaction.
+template <typename T>
+__global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParams p) {
+  constexpr int NW = SPEC_THREADS / 32;
+  __shared__ int32_t s_par[64], s_tok[64];
+  __shared__ int32_t s_path[65];
+  __shared__ int64_t s_src[65], s_dst[65];
+  __shared__ float s_seg[2][SPEC_MAX_SEG];  // per-segment sums of max(0, r - q), double-buffered by rejection
+  __shared__ float s_zk[64];             // Z_1 .. Z_k of the residual at the current node
+  __shared__ float s_rows[4];            // (M, Z) of the current node's target and draft rows
+  __shared__ int s_cmd[4];
+  const int b = blockIdx.x, Tm = p.tr.T_max, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t rb = int64_t(b) * Tm;
+  const int TL = __ldg(p.tr.tree_len + b), L = __ldg(p.tr.kv_len + b);
+  const int64_t V = p.tgt.V;
+  const int nseg = p.tgt.nseg;
+  const float k2 = p.tgt.k2;
+  // the tree's shape needs no statistics: checked while launch 1 runs
+  if (warp == 0) {
+    int bad = 0;
+    if (TL < 1 || TL > Tm) {
+      bad = DREAMS_DATA_BAD_TREE_LEN;
+    } else if (L < 0 || L > p.kv.capacity - TL) {
+      bad = DREAMS_DATA_BAD_KV_LEN;
+    } else {
+      const TreeShape ts = tree_shape_warp(p.tr.parent + rb, p.tr.tokens + rb, TL);
+      bad = ts.bad;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        s_par[lane + 32 * h] = ts.par[h];
+        s_tok[lane + 32 * h] = ts.tok[h];
+      }
+    }
+    if (lane == 0) {
+      s_cmd[0] = bad;
+      if (bad) flag(p.status, bad);
+    }
+  }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  __syncthreads();
+  const int bad = s_cmd[0];
+  int n = -1, bonus = 0;
+  if (!bad) {
+    int cur = 0;
+    n = 0;
+    if (tid == 0) s_path[0] = 0;
+    for (;;) {
+      const int64_t row = rb + cur;
+      const T *trow = static_cast<const T *>(p.tgt.logits) + row * p.tgt.row_stride;
+      const T *drow = static_cast<const T *>(p.drf.logits) + row * p.drf.row_stride;
+      bool kids = false;
+      for (int c = cur + 1; c < TL && !kids; ++c) kids = s_par[c] == cur;
+      const bool try_kids = kids && n < p.max_path - 1;
+      if (warp == 0) {
+        const float2 mz = spec_row_mz(p.tgt.seg + row * nseg, nseg, k2);
+        if (lane == 0) s_rows[0] = mz.x, s_rows[1] = mz.y;
+      } else if (warp == 1 && try_kids) {
+        const float2 mz = spec_row_mz(p.drf.seg + row * nseg, nseg, k2);
+        if (lane == 0) s_rows[2] = mz.x, s_rows[3] = mz.y;
+      }
+      __syncthreads();
+      const float Mt = s_rows[0], Zt = s_rows[1], Md = s_rows[2], Zd = s_rows[3];
+      int k = 0, next = -1;
+      int eff = -1;  // the last rejection whose residual sum was positive (the draw's segment sums)
+      for (int c = cur + 1; c < TL && try_kids; ++c) {
+        if (s_par[c] != cur) continue;
+        if (tid == 0) {
+          const int x = s_tok[c];
+          float a = 0.f;
+          if (x >= 0 && x < V) {
+            const float pv = exp2f_approx((__uint_as_float(Elem<T>::bits(trow, x)) - Mt) * k2) / Zt;
+            const float qv = exp2f_approx((__uint_as_float(Elem<T>::bits(drow, x)) - Md) * k2) / Zd;
+            const float rv = spec_residual(pv, qv, s_zk, k);
+            a = qv > 0.f ? fminf(1.f, rv / qv) : (rv > 0.f ? 1.f : 0.f);
+          }
+          s_cmd[1] = __ldg(p.u_acc + rb + c) < a;
+        }
+        __syncthreads();
+        if (s_cmd[1]) {
+          next = c;
+          break;
+        }
+        // a rejection: the residual's normaliser, and its sums per segment
+        // for a draw from it, in one pass over both rows. After a zero sum
+        // (r == q) the residual is kept, so every later sum at this node is
+        // zero too: no pass, and the sums of the last positive one stay.
+        const bool kept = k > 0 && s_zk[k - 1] == 0.f;
+        for (int g = warp; g < nseg && !kept; g += NW) {
+          float xt[4][8], xd[4][8];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            sub_load<T>(trow, V, p.tgt.vec_ok, 4 * int64_t(g) + j, xt[j]);
+            sub_load<T>(drow, V, p.drf.vec_ok, 4 * int64_t(g) + j, xd[j]);
+          }
+          float acc = 0.f;
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float pv = exp2f_approx((xt[j][e] - Mt) * k2) / Zt;
+              const float qv = exp2f_approx((xd[j][e] - Md) * k2) / Zd;
+              acc += fmaxf(spec_residual(pv, qv, s_zk, k) - qv, 0.f);
+            }
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+          if (lane == 0) s_seg[k & 1][g] = acc;
+        }
+        __syncthreads();
+        if (warp == 0) {
+          float z = 0.f;
+          for (int g = lane; g < nseg && !kept; g += 32) z += s_seg[k & 1][g];
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
+          if (lane == 0) s_zk[k] = z;
+        }
+        __syncthreads();
+        // a zero sum (r == q) keeps the residual, and the sums it was drawn from
+        if (s_zk[k] > 0.f) eff = k;
+        ++k;
+      }
+      if (next >= 0) {
+        ++n;
+        cur = next;
+        if (tid == 0) s_path[n] = next;
+        continue;
+      }
+      // the bonus: a draw from the residual after k rejections (the target
+      // itself when k = 0) by inverse transform, one warp: segment weights in
+      // order up to the crossing, then the crossing segment's values
+      if (warp == 0) {
+        const float u0 = __ldg(p.u_res + rb + cur);
+        const float u = u0 > 0.f ? fminf(u0, 1.f) : 0.f;
+        auto seg_w = [&](int g) -> float {
+          if (g >= nseg) return 0.f;
+          if (eff < 0) {
+            const float2 v = __ldcg(p.tgt.seg + row * nseg + g);
+            return v.x == -INFINITY ? 0.f : v.y * exp2f_approx((v.x - Mt) * k2) / Zt;
+          }
+          return s_seg[eff & 1][g] / s_zk[eff];
+        };
+        int gs = -1, glast = -1;
+        float carry = 0.f, rem = 0.f;
+        for (int base = 0; base < nseg && gs < 0; base += 32) {
+          const float w = seg_w(base + lane);
+          float inc = w;
+#pragma unroll
+          for (int off = 1; off < 32; off <<= 1) {
+            const float y = __shfl_up_sync(0xffffffffu, inc, off);
+            if (lane >= off) inc += y;
+          }
+          const unsigned pos = __ballot_sync(0xffffffffu, w > 0.f);
+          if (pos) glast = base + 31 - __clz(pos);
+          const unsigned cross = __ballot_sync(0xffffffffu, w > 0.f && carry + inc > u);
+          if (cross) {
+            const int l0 = __ffs(cross) - 1;
+            gs = base + l0;
+            rem = u - (carry + __shfl_sync(0xffffffffu, inc - w, l0));
+          }
+          carry += __shfl_sync(0xffffffffu, inc, 31);
+        }
+        const bool tail = gs < 0;  // no crossing (u at the very end): the last value of positive weight
+        if (tail) gs = glast >= 0 ? glast : 0;
+        int pick = -1, lastpos = -1;
+        float acc = 0.f;
+        for (int j = 0; j < 4 && pick < 0; ++j) {
+          float xt[8], xd[8];
+          sub_load<T>(trow, V, p.tgt.vec_ok, 4 * int64_t(gs) + j, xt);
+          sub_load<T>(drow, V, p.drf.vec_ok, 4 * int64_t(gs) + j, xd);
+          float w[8], ls = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float pv = exp2f_approx((xt[e] - Mt) * k2) / Zt;
+            w[e] = k == 0 ? pv : spec_residual(pv, exp2f_approx((xd[e] - Md) * k2) / Zd, s_zk, k);
+            ls += w[e];
+          }
+          float inc = ls;
+#pragma unroll
+          for (int off = 1; off < 32; off <<= 1) {
+            const float y = __shfl_up_sync(0xffffffffu, inc, off);
+            if (lane >= off) inc += y;
+          }
+          const int64_t e0 = int64_t(gs) * SEG + j * SUB + 8 * lane;
+          int lp = -1;
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            if (w[e] > 0.f) lp = int(e0) + e;
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, off));
+          if (lp >= 0) lastpos = lp;
+          if (!tail) {
+            const unsigned cross = __ballot_sync(0xffffffffu, acc + inc > rem && ls > 0.f);
+            if (cross) {
+              const int l0 = __ffs(cross) - 1;
+              int hit = -1;
+              if (lane == l0) {
+                float a = acc + inc - ls;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  a += w[e];
+                  if (hit < 0 && w[e] > 0.f && a > rem) hit = int(e0) + e;
+                }
+                if (hit < 0) hit = lp;  // rounding: the last positive value of this lane's 8
+              }
+              pick = __shfl_sync(0xffffffffu, hit, l0);
+            }
+          }
+          acc += __shfl_sync(0xffffffffu, inc, 31);
+        }
+        if (pick < 0) pick = lastpos >= 0 ? lastpos : 0;
+        if (lane == 0) s_cmd[2] = int(std::min<int64_t>(std::max(pick, 0), V - 1));
+      }
+      __syncthreads();
+      bonus = s_cmd[2];
+      break;
+    }
+  }
+  // outputs: path, drafts then the bonus, lengths (warp 0)
+  if (warp == 0) {
+    const int mp = p.max_path;
+    for (int kk = lane; kk < mp; kk += 32) {
+      int pv = -1, ov = -1;
+      if (n >= 0 && kk <= n) {
+        pv = s_path[kk];
+        ov = kk < n ? s_tok[s_path[kk + 1]] : bonus;
+      }
+      p.path[int64_t(b) * mp + kk] = pv;
+      p.out_tokens[int64_t(b) * mp + kk] = ov;
+    }
+    if (lane == 0) {
+      p.accept_len[b] = n >= 0 ? n + 1 : 0;
+      p.new_kv_len[b] = n >= 0 ? L + n + 1 : L;
+    }
+    bool ok = n > 0;
+    if (ok) ok = move_offsets(p.kv, b, L, n, s_path, s_src, s_dst, p.status);
+    if (lane == 0) s_cmd[3] = ok ? n : 0;
+  }
+  __syncthreads();
+  const int nm = s_cmd[3];
+  if (nm > 0) compact_units(p.kv, nm, s_src, s_dst, tid, SPEC_THREADS);
+}
+
 // ------------------------------------------------------------------ host side
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -1332,6 +1661,58 @@ extern "C" dreams_status_t dreams_verify_step_sampled(
                            : launch_dependent(verify_sample_select_kernel<__nv_bfloat16>, g2, dim3(256), s, p);
   if (st != DREAMS_OK) return st;
   return launch_dependent(verify_tail_kernel, dim3(unsigned(tree->B)), dim3(TAIL_THREADS), s, p);
+}
+
+extern "C" size_t dreams_verify_step_speculative_workspace_size(const dreams_tree_t *tree, int64_t V) {
+  if (tree == nullptr || tree->B < 1 || tree->T_max < 1 || tree->T_max > 64 || V < 1) return 0;
+  const int64_t rows = int64_t(tree->B) * tree->T_max;
+  return 2 * sample_ws(rows, V);
+}
+
+extern "C" dreams_status_t dreams_verify_step_speculative(
+    const void *target_logits, const void *draft_logits, dreams_dtype_t dtype, int64_t V, int64_t row_stride,
+    const dreams_tree_t *tree, const dreams_kv_cache_t *kv, int32_t max_path, float temperature,
+    const float *u_accept, const float *u_resample, int32_t *accept_len, int32_t *path, int32_t *out_tokens,
+    int32_t *new_kv_len, void *workspace, size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream) {
+  SpecParams p{};
+  if (target_logits == nullptr || draft_logits == nullptr || u_accept == nullptr || u_resample == nullptr || V < 1 ||
+      V > INT_MAX - SEG || row_stride < V || !tree_params(tree, true, p.tr) || !kv_params(kv, p.kv) ||
+      max_path < 1 || max_path > 65 || accept_len == nullptr || path == nullptr || out_tokens == nullptr ||
+      new_kv_len == nullptr)
+    return DREAMS_ERR_INVALID_ARG;
+  if (dtype != DREAMS_F32 && dtype != DREAMS_BF16) return DREAMS_ERR_UNSUPPORTED;
+  const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
+  if (reinterpret_cast<uintptr_t>(target_logits) % esz || reinterpret_cast<uintptr_t>(draft_logits) % esz ||
+      (reinterpret_cast<uintptr_t>(u_accept) & 3) || (reinterpret_cast<uintptr_t>(u_resample) & 3))
+    return DREAMS_ERR_INVALID_ARG;
+  if ((V + SEG - 1) / SEG > SPEC_MAX_SEG) return DREAMS_ERR_UNSUPPORTED;
+  const int64_t rows = int64_t(tree->B) * tree->T_max;
+  const size_t need = dreams_verify_step_speculative_workspace_size(tree, V);
+  if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace)) return DREAMS_ERR_WORKSPACE;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  int64_t ctas = 0, ctas_d = 0;
+  if (!sample_params(target_logits, dtype, rows, V, row_stride, temperature, u_resample, ws, p.tgt, ctas) ||
+      !sample_params(draft_logits, dtype, rows, V, row_stride, temperature, u_resample, ws + sample_ws(rows, V), p.drf,
+                     ctas_d))
+    return DREAMS_ERR_INVALID_ARG;
+  if (2 * ctas > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  p.max_path = max_path;
+  p.u_acc = u_accept;
+  p.u_res = u_resample;
+  p.accept_len = accept_len;
+  p.path = path;
+  p.out_tokens = out_tokens;
+  p.new_kv_len = new_kv_len;
+  p.status = status_word;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const dim3 grid(static_cast<unsigned>(2 * ctas));
+  if (dtype == DREAMS_F32) spec_stats_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  else spec_stats_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
+  const dreams_status_t st = check_launch();
+  if (st != DREAMS_OK) return st;
+  return dtype == DREAMS_F32
+             ? launch_dependent(spec_walk_kernel<float>, dim3(unsigned(tree->B)), dim3(SPEC_THREADS), s, p)
+             : launch_dependent(spec_walk_kernel<__nv_bfloat16>, dim3(unsigned(tree->B)), dim3(SPEC_THREADS), s, p);
 }
 
 // ------------------------------------------------------------------ no-allocation argmax
