@@ -102,6 +102,21 @@ def speculative_bytes(w: W.Workload) -> int:
     return argmax_bytes(w) + inner * w.V * (4 if w.logits_dtype == "f32" else 2)
 
 
+def speculative_visited_bytes(w: W.Workload, accept_len, path, max_path: int) -> int:
+    """Bytes of the rows the speculative walk needs: the target row of every
+    node on the walked path, and the draft row of each of those nodes whose
+    children were tried (it has children and the walk was not cut there)."""
+    esz = 4 if w.logits_dtype == "f32" else 2
+    rows = 0
+    for b in range(w.B):
+        par = w.parent[b, :int(w.tree_len[b])].numpy()
+        inner = set(int(x) for x in par[1:])
+        for kk in range(int(accept_len[b])):
+            node = int(path[b, kk])
+            rows += 1 + int(node in inner and kk < max_path - 1)
+    return rows * w.V * esz
+
+
 def attn_flops(w: W.Workload) -> int:
     return int(sum(4 * int(w.tree_len[b]) * w.Hq * (int(w.kv_len[b]) + int(w.tree_len[b])) * w.D
                    for b in range(w.B)))
@@ -517,35 +532,48 @@ def run_dreams(args, rank, world, local):
         cpu_g = torch.Generator().manual_seed(13)
         u_a = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
         u_r = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
-        ws_sp = torch.zeros(dreams.verify_step_speculative_workspace_size(copies[0]["tree"], w.V),
-                            dtype=torch.uint8, device=dev)
 
         def spec_call(i):
             c = copies[i % 2]
             dreams.verify_step_speculative(c["logits"], drafts[i % 2], c["tree"], c["kv"], max_path, 1.0, u_a, u_r,
-                                           outputs=c["outs"], workspace=ws_sp, status=status)
+                                           outputs=c["outs"], status=status)
 
         for i in range(4):
             spec_call(i)
+        spec_graphs, spec_mode = None, "eager"
+        if not args.no_graph:
+            spec_graphs = []
+            for i in range(2):
+                gsp = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gsp):
+                    spec_call(i)
+                spec_graphs.append(gsp)
+            spec_mode = "cuda-graph replay"
         Ks = max(3, min(K, 100))
         s0 = torch.cuda.Event(enable_timing=True)
         s1 = torch.cuda.Event(enable_timing=True)
         barrier()
         s0.record(stream)
         for i in range(Ks):
-            spec_call(i)
+            if spec_graphs is not None:
+                spec_graphs[i % 2].replay()
+            else:
+                spec_call(i)
         s1.record(stream)
         barrier()
         if int(status.item()) != 0:
             raise RuntimeError(f"device status {int(status.item()):#x} on valid input (speculative step)")
-        acc_mean = float(copies[(Ks - 1) % 2]["outs"][0].float().mean())
+        outs = copies[(Ks - 1) % 2]["outs"]
+        acc_np, path_np = outs[0].cpu().numpy(), outs[1].cpu().numpy()
         spec_us = s0.elapsed_time(s1) / Ks * 1000.0
-        sb = speculative_bytes(w)
+        vb = speculative_visited_bytes(w, acc_np, path_np, max_path)
         speculative = {"us": round(spec_us, 2), "temperature": 1.0,
-                       "launches": dreams.VERIFY_STEP_SPECULATIVE_LAUNCHES, "launch": "eager",
-                       "bytes": sb, "GBps": round(sb / (spec_us * 1e-6) / 1e9, 1),
-                       "draft": "target logits + N(0, 0.5) noise", "mean_accept_len": round(acc_mean, 3)}
-        del drafts
+                       "launches": dreams.VERIFY_STEP_SPECULATIVE_LAUNCHES, "launch": spec_mode,
+                       "visited_row_bytes": vb, "GBps": round(vb / (spec_us * 1e-6) / 1e9, 1),
+                       "all_rows_bytes": speculative_bytes(w),
+                       "draft": "target logits + N(0, 0.5) noise",
+                       "mean_accept_len": round(float(acc_np.mean()), 3)}
+        del drafts, spec_graphs
 
     # ---- the LM head with its argmax fused (the logits never reach HBM), on
     # the tree rows of this workload: hidden size Hq * D, random bf16 weights

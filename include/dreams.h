@@ -318,28 +318,28 @@ dreams_status_t dreams_verify_step_sampled(const void *logits, dreams_dtype_t dt
  * clamped to [0, 1]; none: the last v of positive weight). accept_len, path,
  * out_tokens, new_kv_len and the KV compaction are as in dreams_verify_step.
  * target_logits, draft_logits: f32 or bf16, [B, T_max, V] with row_stride
- * (the same for both); the draft rows of leaves are not read. u_accept,
- * u_resample: device f32 [B, T_max] (the caller's random numbers). Logits must
- * be finite (with non-finite values the tokens drawn are unspecified but lie in
- * [0, V)). V <= 524288, max_path <= 65. Arithmetic is f32 (hardware exp2 of the
- * scaled differences), so a decision can differ from the exact-arithmetic one
- * only when a uniform lies within rounding of its threshold. Two launches,
- * chained by programmatic dependent launch: the 1024-value segment statistics
- * of the target rows of the tree nodes and of the draft rows of nodes with
- * children (8 bytes per 1024 values per row in the workspace); then one CTA
- * per sequence that walks the tree, taking one pass over both rows of a node
- * for each rejection there (the residual's sum), draws the bonus, writes the
- * outputs and moves the accepted K/V. The workspace holds no state between
- * calls.
+ * (the same for both); only the rows of the nodes the walk visits are read
+ * (the draft row only where children are tried). u_accept, u_resample:
+ * device f32 [B, T_max] (the caller's random numbers). Logits must be finite
+ * (with non-finite values the tokens drawn are unspecified but lie in
+ * [0, V)). V <= 393216 (beyond 196608 the kernel needs clusters of 16 CTAs),
+ * max_path <= 65. Arithmetic is f32 (hardware exp2 of the scaled
+ * differences), so a decision can differ from the exact-arithmetic one only
+ * when a uniform lies within rounding of its threshold. The kernel holds the
+ * residual in closed form, r = max(0, p - s q) / P with P = sum_v max(0, p -
+ * s q) (s = 0 at the node; a rejection sets s to s + P), which is the
+ * recursion above. One launch, no workspace: a cluster of up to 16 CTAs per
+ * sequence, each holding a slice of the visited node's rows in shared memory;
+ * a rejection costs one sum over the slices, combined across the cluster in
+ * distributed shared memory. The cluster then draws the bonus, writes the
+ * outputs and moves the accepted K/V.
  */
-size_t dreams_verify_step_speculative_workspace_size(const dreams_tree_t *tree, int64_t V);
 dreams_status_t dreams_verify_step_speculative(const void *target_logits, const void *draft_logits,
                                                dreams_dtype_t dtype, int64_t V, int64_t row_stride,
                                                const dreams_tree_t *tree, const dreams_kv_cache_t *kv,
                                                int32_t max_path, float temperature, const float *u_accept,
                                                const float *u_resample, int32_t *accept_len, int32_t *path,
-                                               int32_t *out_tokens, int32_t *new_kv_len, void *workspace,
-                                               size_t workspace_bytes, int32_t *status_word,
+                                               int32_t *out_tokens, int32_t *new_kv_len, int32_t *status_word,
                                                dreams_stream_t stream);
 
 /*

@@ -102,9 +102,8 @@ def _lib() -> ctypes.CDLL:
                     "dreams_verify_step_sampled_workspace_size": (sz, [ptr, i64]),
                     "dreams_verify_step_sampled": (ctypes.c_int, [p, ctypes.c_int, i64, i64, ptr, pkv, i32, f32, p,
                                                                   p, p, p, p, p, p, sz, p, p]),
-                    "dreams_verify_step_speculative_workspace_size": (sz, [ptr, i64]),
                     "dreams_verify_step_speculative": (ctypes.c_int, [p, p, ctypes.c_int, i64, i64, ptr, pkv, i32,
-                                                                      f32, p, p, p, p, p, p, p, sz, p, p]),
+                                                                      f32, p, p, p, p, p, p, p, p]),
                     "dreams_test_set_stall": (ctypes.c_int, [i32, i32, i64]),
                     "dreams_status_string": (ctypes.c_char_p, [ctypes.c_int]),
                     "dreams_version": (i32, []),
@@ -502,10 +501,6 @@ def verify_step_sampled_workspace_size(tree: Tree, V: int) -> int:
     return int(_lib().dreams_verify_step_sampled_workspace_size(ctypes.byref(tree._c), V))
 
 
-def verify_step_speculative_workspace_size(tree: Tree, V: int) -> int:
-    return int(_lib().dreams_verify_step_speculative_workspace_size(ctypes.byref(tree._c), V))
-
-
 def verify_step_workspace_size(tree: Tree, V: int) -> int:
     return int(_lib().dreams_verify_step_workspace_size(ctypes.byref(tree._c), V))
 
@@ -570,11 +565,11 @@ def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path:
 
 def verify_step_speculative(target_logits: torch.Tensor, draft_logits: torch.Tensor, tree: Tree, kv: KVCache,
                             max_path: int, temperature: float, u_accept: torch.Tensor, u_resample: torch.Tensor,
-                            outputs: Optional[tuple] = None, workspace: Optional[torch.Tensor] = None,
-                            status: Optional[torch.Tensor] = None, stream=None) -> dict:
+                            outputs: Optional[tuple] = None, status: Optional[torch.Tensor] = None,
+                            stream=None) -> dict:
     """The verification tail at temperature > 0 by speculative sampling over
-    the tree: a draft is accepted with probability min(1, p/q) against the
-    current residual, a rejection renormalises max(0, p - q), and the bonus is
+    the tree: a draft is accepted with probability min(1, r/q) against the
+    current residual r, a rejection renormalises max(0, r - q), and the bonus is
     drawn from what is left (``dreams_verify_step_speculative``). target_logits
     and draft_logits: [B, T_max, V] f32/bf16 with the same strides; u_accept,
     u_resample: f32 [B, T_max]. Then acceptance outputs and KV compaction."""
@@ -594,17 +589,15 @@ def verify_step_speculative(target_logits: torch.Tensor, draft_logits: torch.Ten
             raise ValueError(f"{n} must be [B, T_max]")
     V = int(target_logits.shape[2])
     acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
-    if workspace is None:
-        workspace = _workspace("step_speculative", verify_step_speculative_workspace_size(tree, V), dev, stream)
     _call("dreams_verify_step_speculative", dev,
           _ptr(target_logits), _ptr(draft_logits), F32 if target_logits.dtype == torch.float32 else BF16, V,
           int(target_logits.stride(1)), ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature),
-          _ptr(u_accept), _ptr(u_resample), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(workspace),
-          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
+          _ptr(u_accept), _ptr(u_resample), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(status),
+          _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
 
-VERIFY_STEP_SPECULATIVE_LAUNCHES = 2  # segment statistics, then the walk with its passes and the compaction
+VERIFY_STEP_SPECULATIVE_LAUNCHES = 1  # one cluster per sequence: walk, residual sums, bonus, compaction
 
 
 def test_set_stall(kernels: int, stall_at: int, wait_limit_ns: int = 20_000_000) -> None:

@@ -2,7 +2,7 @@
 // CUDA error, and the cached SM count used to size grids.
 #include <atomic>
 #include <mutex>
-#include <set>
+#include <map>
 #include <utility>
 
 #include "common.cuh"
@@ -14,7 +14,7 @@ thread_local int32_t g_last_cuda_error = 0;
 std::mutex g_sm_mutex;
 int g_sm_count[64] = {0};
 std::mutex g_attr_mutex;
-std::set<std::pair<const void *, int>> g_attr_done;  // (kernel, device) pairs configured
+std::map<std::pair<const void *, int>, int> g_attr_done;  // (kernel, device) -> the largest limit set
 constexpr uint64_t DEFAULT_WAIT_NS = 2000000000ull;
 std::atomic<int32_t> g_stall_kernels{0};
 std::atomic<int32_t> g_stall_at{-1};
@@ -53,13 +53,14 @@ dreams_status_t ensure_max_dynamic_smem(const void *func, int bytes) {
     return DREAMS_ERR_CUDA;
   }
   std::lock_guard<std::mutex> lock(g_attr_mutex);
-  if (g_attr_done.count({func, dev})) return DREAMS_OK;
+  const auto it = g_attr_done.find({func, dev});
+  if (it != g_attr_done.end() && it->second >= bytes) return DREAMS_OK;
   e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return DREAMS_ERR_CUDA;
   }
-  g_attr_done.insert({func, dev});
+  g_attr_done[{func, dev}] = bytes;
   return DREAMS_OK;
 }
 

@@ -16,8 +16,9 @@ void set_last_cuda_error(cudaError_t e);
 // Streaming multiprocessors of the current device (cached per device).
 int num_sms();
 
-// Sets a kernel's maximum dynamic shared memory on the current device, once
-// per (kernel, device); safe to call from several host threads.
+// Raises a kernel's maximum dynamic shared memory on the current device to at
+// least `bytes` (the attribute is set again only for a larger request); safe
+// to call from several host threads.
 dreams_status_t ensure_max_dynamic_smem(const void *func, int bytes);
 
 // The stall test hook (dreams_test_set_stall) as it applies to one kernel

@@ -1021,11 +1021,38 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
 // min(1, r(x) / q(x)); a rejection replaces r by max(0, r - q) / Z with
 // Z = sum max(0, r - q) (kept when Z = 0). The bonus is drawn from r by
 // inverse transform with u_res of the node where the walk stops.
-constexpr int SPEC_THREADS = 512;     // walk kernel: 16 warps share the passes over a row
-constexpr int SPEC_MAX_SEG = 512;     // 1024-value segments per row the walk keeps sums of (V <= 524288)
+//
+// The kernel keeps r in closed form. With r = max(0, p - s q) / P, where
+// P = F(s) = sum_v max(0, p_v - s q_v) (s = 0, P = 1: r = p), a rejection gives
+// max(0, r - q) = max(0, p - (s + P) q) / P (where p - s q <= 0 the term is 0
+// either way), so the next residual is max(0, p - s' q) / F(s') with
+// s' = s + P, and Z = F(s') / P. In the unnormalised exponentials
+// e_v = 2^((x_v - M) k2) of the two rows (sums Zt, Zd) this reads
+//     r ~ max(0, et - c ed),  Pu = sum_v max(0, et_v - c ed_v),
+//     c = 0, Pu = Zt at the node;  a rejection: c' = c + Pu / Zd,
+//     a child with draft x: accepted when u < Zd max(0, et_x - c ed_x) / (Pu ed_x)
+// (c = s Zt / Zd, Pu = Zt P): one sum over the vocabulary per rejection, and
+// the bonus is drawn from the weights max(0, et - c ed) (et when c = 0).
+//
+// One thread-block cluster per sequence; CTA `rank` of the cluster holds the
+// vocabulary slice [rank * S, (rank + 1) * S) of the rows of the node being
+// visited, as exponentials in shared memory. Only the rows of visited nodes
+// are read. A sum (or maximum) over the vocabulary: every warp reduces its
+// threads' values and stores the result into every CTA's shared memory
+// (distributed shared memory), one cluster barrier, then each warp combines
+// the cs * 16 values in the same fixed order: all CTAs hold bit-identical
+// results, take the same decisions and pass the same cluster barriers.
+constexpr int SPEC_THREADS = 512;                    // 16 warps
+constexpr int SPEC_CHUNK = 8 * SPEC_THREADS;         // values per chunk: 8 per thread
+constexpr int SPEC_MAX_J = 6;                        // chunks per CTA slice (192 KB of f32 pairs)
+constexpr int SPEC_MAX_CS = 16;                      // CTAs per cluster
 
 struct SpecParams {
-  SampleParams tgt, drf;  // 1024-value segment statistics (m, sum 2^((x - m) k2)) of target and draft rows
+  const void *tgt, *drf;  // [B * T_max] rows of V logits, row_stride apart
+  int64_t V, row_stride;
+  float k2;               // log2(e) / tau
+  int vec_ok;             // rows start on 16 bytes and strides keep them there
+  int cs, J;              // CTAs per cluster, chunks per slice
   TreeParams tr;
   KVParams kv;
   int32_t max_path;
@@ -1034,89 +1061,307 @@ struct SpecParams {
   int32_t *status;
 };
 
-// Launch 1: statistics of the target rows of the tree nodes and of the draft
-// rows of nodes that have children. grid.x = 2 * B * T_max * ncta_row: (row
-// set, node row, CTA of the row); rows that are not needed return at once.
-template <typename T>
-__global__ void __launch_bounds__(SAMPLE_THREADS, sizeof(T) == 2 ? 6 : 4) spec_stats_kernel(const SpecParams p) {
-  const int ncta = p.tgt.ncta_row;
-  const int64_t rows = int64_t(p.tr.B) * p.tr.T_max;
-  const int64_t x = blockIdx.x / ncta;
-  const bool drf = x >= rows;
-  const int64_t r = drf ? x - rows : x;
-  const int b = int(r / p.tr.T_max), i = int(r % p.tr.T_max);
-  const int tl = __ldg(p.tr.tree_len + b);
-  bool live = tl >= 1 && tl <= p.tr.T_max && i < tl;
-  if (live && drf) {  // only a node with children has a draft distribution to read
-    bool kids = false;
-    for (int c = i + 1; c < tl && !kids; ++c) kids = __ldg(p.tr.parent + int64_t(b) * p.tr.T_max + c) == i;
-    live = kids;
-  }
-  if (live) {
-    const SampleParams &sp = drf ? p.drf : p.tgt;
-    const int64_t g0 = int64_t(blockIdx.x % ncta) * sp.seg_per_cta;
-    const int64_t g1 = std::min<int64_t>(sp.nseg, g0 + sp.seg_per_cta);
-    sample_stats<T>(sp, static_cast<const T *>(sp.logits) + r * sp.row_stride, sp.seg + r * sp.nseg, g0, g1);
-  }
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-
-// (M, Z) of a row from its segment statistics, Z = sum_v 2^((x_v - M) k2); one
-// warp. The statistics were written by the preceding grid: read through L2.
-__device__ float2 spec_row_mz(const float2 *seg_row, int nseg, float k2) {
-  const int lane = threadIdx.x & 31;
-  float m_l = -INFINITY, z_l = 0.f;
-  for (int g = lane; g < nseg; g += 32) {
-    const float2 v = __ldcg(seg_row + g);
-    if (v.x == -INFINITY) continue;
-    if (v.x > m_l) {
-      z_l = (m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - v.x) * k2)) + v.y;
-      m_l = v.x;
-    } else {
-      z_l += v.y * exp2f_approx((v.x - m_l) * k2);
-    }
-  }
-  float M = m_l;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-  float Z = m_l == -INFINITY ? 0.f : z_l * exp2f_approx((m_l - M) * k2);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) Z += __shfl_xor_sync(0xffffffffu, Z, off);
-  return make_float2(M, Z);
-}
-
-// The residual after k rejections at a node, at one vocabulary entry, from
-// the target and draft probabilities there: r_0 = p, r_j = max(0, r_{j-1} - q) /
-// Z_j (kept when Z_j = 0).
-__device__ __forceinline__ float spec_residual(float pv, float qv, const float *zk, int k) {
-  float r = pv;
-  for (int j = 0; j < k; ++j) {
-    const float z = zk[j];
-    if (z > 0.f) r = fmaxf(r - qv, 0.f) / z;
-  }
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
 
-// Launch 2, one CTA per sequence (chained to launch 1 by programmatic
-// dependent launch): the walk with its decisions, the bonus draw, the outputs
-// and the KV compaction.
+// Every thread of every CTA of the cluster: release this CTA's shared-memory
+// writes (local and remote), then wait for all CTAs (a superset of
+// __syncthreads).
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_addr(const void *local_ptr, uint32_t rank) {
+  const uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(local_ptr));
+  uint32_t ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+  return ra;
+}
+__device__ __forceinline__ void st_cluster_f2(const float2 *local_ptr, uint32_t rank, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(cluster_addr(local_ptr, rank)), "f"(v.x), "f"(v.y)
+               : "memory");
+}
+__device__ __forceinline__ void st_cluster_s32(const int32_t *local_ptr, uint32_t rank, int32_t v) {
+  asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(cluster_addr(local_ptr, rank)), "r"(v) : "memory");
+}
+
+struct SpecShared {
+  float2 slot[2][SPEC_MAX_CS * 16];  // [parity][rank * 16 + warp]: every warp's partial of every CTA
+  float chunk[SPEC_MAX_J][16];       // the bonus draw: per-warp sums of each chunk
+  int32_t hit[16], last[16];
+  int32_t par[64], tok[64], path[65];
+  int64_t src[65], dst[65];
+  float cet[64], ced[64];  // exponentials of the target / draft logits at each child's draft token
+  float cu[64];            // u_acc of each child
+  int32_t pick;            // the draw inside this CTA's slice
+  int32_t bonus;           // rank 0: the bonus token, written by the CTA that drew it
+  int32_t cmd;
+};
+
+struct SpecMax {
+  __device__ static float f(float a, float b) { return fmaxf(a, b); }
+  __device__ static float id() { return -INFINITY; }
+};
+struct SpecSum {
+  __device__ static float f(float a, float b) { return a + b; }
+  __device__ static float id() { return 0.f; }
+};
+
+// Each warp reduces its threads' pairs and stores the result into slot
+// [parity][rank * 16 + warp] of every CTA of the cluster; then the cluster
+// barrier. No thread reads another CTA's memory afterwards.
+template <class Op>
+__device__ __forceinline__ void spec_push(SpecShared &sh, float2 v, int parity, int cs, uint32_t rank) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    v.x = Op::f(v.x, __shfl_xor_sync(0xffffffffu, v.x, off));
+    v.y = Op::f(v.y, __shfl_xor_sync(0xffffffffu, v.y, off));
+  }
+  v.x = __shfl_sync(0xffffffffu, v.x, 0);  // lane 0's bits on every lane
+  v.y = __shfl_sync(0xffffffffu, v.y, 0);
+  if (lane < cs) st_cluster_f2(&sh.slot[parity][rank * 16 + warp], uint32_t(lane), v);
+  cluster_sync();
+}
+
+// The combination of all cs * 16 pushed pairs in the same fixed order in every
+// warp of every CTA, so the bits agree everywhere.
+template <class Op>
+__device__ __forceinline__ float2 spec_combine(const SpecShared &sh, int parity, int cs) {
+  const int lane = threadIdx.x & 31;
+  float2 acc = make_float2(Op::id(), Op::id());
+  for (int i = lane; i < cs * 16; i += 32) {
+    const float2 v = sh.slot[parity][i];
+    acc.x = Op::f(acc.x, v.x);
+    acc.y = Op::f(acc.y, v.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    acc.x = Op::f(acc.x, __shfl_xor_sync(0xffffffffu, acc.x, off));
+    acc.y = Op::f(acc.y, __shfl_xor_sync(0xffffffffu, acc.y, off));
+  }
+  acc.x = __shfl_sync(0xffffffffu, acc.x, 0);
+  acc.y = __shfl_sync(0xffffffffu, acc.y, 0);
+  return acc;
+}
+
+// This thread's values of one slice as floats into e (values past V: -inf);
+// returns their maximum.
+template <typename T>
+__device__ __forceinline__ float spec_store_raw(const SpecParams &p, const uint4 (&w)[SPEC_MAX_J][sizeof(T) / 2],
+                                                float *e) {
+  constexpr int NW = int(sizeof(T)) / 2;  // 16-byte words per 8 values
+  const int tid = threadIdx.x;
+  float m = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j)
+    if (j < p.J) {
+      float y[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        y[i] = __uint_as_float(Elem<T>::lane_bits(w[j][NW == 1 ? 0 : i >> 2], NW == 1 ? i : (i & 3)));
+        m = fmaxf(m, y[i]);
+      }
+      float4 *dst = reinterpret_cast<float4 *>(e + j * SPEC_CHUNK + 8 * tid);
+      dst[0] = make_float4(y[0], y[1], y[2], y[3]);
+      dst[1] = make_float4(y[4], y[5], y[6], y[7]);
+    }
+  return m;
+}
+
+// This CTA's slices of the target row (and of the draft row when `both`) as
+// floats into et / ed; this thread's maxima of each. bf16 rows have both
+// rows' loads in flight at once; f32 rows are taken one after the other.
+template <typename T>
+__device__ float2 spec_load_rows(const SpecParams &p, const T *trow, const T *drow, bool both, int64_t v0, float *et,
+                                 float *ed) {
+  constexpr int NW = int(sizeof(T)) / 2;
+  const int warp = threadIdx.x >> 5;
+  const int64_t Vs = p.V - v0;  // values of the row from the slice start on
+  float2 m = make_float2(-INFINITY, -INFINITY);
+  uint4 wt[SPEC_MAX_J][NW];
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j)
+    if (j < p.J) sub_words<T>(trow + v0, Vs, p.vec_ok, int64_t(j) * (SPEC_CHUNK / SUB) + warp, wt[j]);
+  if (NW == 1) {
+    uint4 wd[SPEC_MAX_J][NW];
+#pragma unroll
+    for (int j = 0; j < SPEC_MAX_J; ++j)
+      if (both && j < p.J) sub_words<T>(drow + v0, Vs, p.vec_ok, int64_t(j) * (SPEC_CHUNK / SUB) + warp, wd[j]);
+    m.x = spec_store_raw<T>(p, wt, et);
+    if (both) m.y = spec_store_raw<T>(p, wd, ed);
+  } else {
+    m.x = spec_store_raw<T>(p, wt, et);
+    if (both) {
+#pragma unroll
+      for (int j = 0; j < SPEC_MAX_J; ++j)
+        if (j < p.J) sub_words<T>(drow + v0, Vs, p.vec_ok, int64_t(j) * (SPEC_CHUNK / SUB) + warp, wt[j]);
+      m.y = spec_store_raw<T>(p, wt, ed);
+    }
+  }
+  return m;
+}
+
+// e <- 2^((e - M) k2) in place over this thread's values; returns their sum.
+__device__ __forceinline__ float spec_exp_inplace(float *e, float M, float k2, int J) {
+  const int tid = threadIdx.x;
+  float s0 = 0.f, s1 = 0.f;
+  for (int j = 0; j < J; ++j) {
+    float4 *q = reinterpret_cast<float4 *>(e + j * SPEC_CHUNK + 8 * tid);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float4 v = q[h];
+      v.x = exp2f_approx((v.x - M) * k2);
+      v.y = exp2f_approx((v.y - M) * k2);
+      v.z = exp2f_approx((v.z - M) * k2);
+      v.w = exp2f_approx((v.w - M) * k2);
+      q[h] = v;
+      s0 += v.x + v.y;
+      s1 += v.z + v.w;
+    }
+  }
+  return s0 + s1;
+}
+
+// The residual's numerator at one vocabulary entry: max(0, et - c ed).
+__device__ __forceinline__ float spec_w(float et, float ed, float c) { return fmaxf(fmaf(-c, ed, et), 0.f); }
+
+// Sum of the residual's numerator over this thread's values (et alone when
+// use_q is false); per chunk into wj, and the last index of positive weight.
+__device__ __forceinline__ float spec_weights(const float *et, const float *ed, float c, bool use_q, int J,
+                                              float (&wj)[SPEC_MAX_J], int &last) {
+  const int tid = threadIdx.x;
+  float tot = 0.f;
+  last = -1;
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j) {
+    wj[j] = 0.f;
+    if (j < J) {
+      const int e0 = j * SPEC_CHUNK + 8 * tid;
+      const float4 *t4 = reinterpret_cast<const float4 *>(et + e0);
+      const float4 *d4 = reinterpret_cast<const float4 *>(ed + e0);
+      float w[8];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const float4 tv = t4[h];
+        if (use_q) {
+          const float4 dv = d4[h];
+          w[4 * h] = spec_w(tv.x, dv.x, c), w[4 * h + 1] = spec_w(tv.y, dv.y, c);
+          w[4 * h + 2] = spec_w(tv.z, dv.z, c), w[4 * h + 3] = spec_w(tv.w, dv.w, c);
+        } else {
+          w[4 * h] = tv.x, w[4 * h + 1] = tv.y, w[4 * h + 2] = tv.z, w[4 * h + 3] = tv.w;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        wj[j] += w[i];
+        if (w[i] > 0.f) last = e0 + i;
+      }
+      tot += wj[j];
+    }
+  }
+  return tot;
+}
+
+// The bonus draw inside this CTA's slice: the entry where the running sum of
+// the weights (in vocabulary order) first exceeds rem; tail: the last entry
+// of positive weight. Returns the slice-relative index (-1: no positive
+// weight) on every thread of the CTA.
+__device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed, float c, bool use_q,
+                               const float (&wj)[SPEC_MAX_J], int last, int J, float rem, bool tail) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, off));
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j) {
+    float v = j < J ? wj[j] : 0.f;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0 && j < J) sh.chunk[j][warp] = v;
+  }
+  if (lane == 0) sh.last[warp] = last;
+  __syncthreads();
+  int slast = -1;
+  for (int w = 0; w < 16; ++w) slast = max(slast, sh.last[w]);
+  if (tail || slast < 0) return slast;
+  // the crossing chunk (every thread walks the same sums in the same order)
+  int jc = -1;
+  float before = 0.f;
+  for (int j = 0; j < J && jc < 0; ++j) {
+    float t = 0.f;
+    for (int w = 0; w < 16; ++w) t += sh.chunk[j][w];
+    if (t > 0.f && before + t > rem) jc = j;
+    else before += t;
+  }
+  if (jc < 0) return slast;  // rounding: no crossing inside the slice
+  rem -= before;
+  // exclusive scan of the threads' sums of chunk jc, in thread order
+  float mine = 0.f;
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j)
+    if (j == jc) mine = wj[j];
+  float inc = mine;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, inc, off);
+    if (lane >= off) inc += y;
+  }
+  float wbase = 0.f;
+  for (int w = 0; w < warp; ++w) wbase += sh.chunk[jc][w];
+  const float excl = wbase + inc - mine;
+  const bool cross = mine > 0.f && excl + mine > rem;
+  const unsigned bal = __ballot_sync(0xffffffffu, cross);
+  if (lane == 0) sh.hit[warp] = bal ? warp * 32 + __ffs(bal) - 1 : INT_MAX;
+  __syncthreads();
+  int th = INT_MAX;
+  for (int w = 0; w < 16; ++w) th = min(th, sh.hit[w]);
+  if (th == INT_MAX) return slast;
+  if (tid == th) {
+    const int e0 = jc * SPEC_CHUNK + 8 * tid;
+    float a = excl;
+    int hit = -1, lp = -1;
+    for (int i = 0; i < 8; ++i) {
+      const float w = use_q ? spec_w(et[e0 + i], ed[e0 + i], c) : et[e0 + i];
+      a += w;
+      if (w > 0.f) lp = e0 + i;
+      if (hit < 0 && w > 0.f && a > rem) hit = e0 + i;
+    }
+    sh.pick = hit >= 0 ? hit : lp;
+  }
+  __syncthreads();
+  return sh.pick;
+}
+
+// One cluster of p.cs CTAs per sequence (grid.x = B * cs): the walk with its
+// decisions, the bonus draw, the outputs and the KV compaction.
 template <typename T>
 __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParams p) {
-  constexpr int NW = SPEC_THREADS / 32;
-  __shared__ int32_t s_par[64], s_tok[64];
-  __shared__ int32_t s_path[65];
-  __shared__ int64_t s_src[65], s_dst[65];
-  __shared__ float s_seg[2][SPEC_MAX_SEG];  // per-segment sums of max(0, r - q), double-buffered by rejection
-  __shared__ float s_zk[64];             // Z_1 .. Z_k of the residual at the current node
-  __shared__ float s_rows[4];            // (M, Z) of the current node's target and draft rows
-  __shared__ int s_cmd[4];
-  const int b = blockIdx.x, Tm = p.tr.T_max, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  extern __shared__ __align__(16) float spec_dyn[];
+  __shared__ SpecShared sh;
+  const int cs = p.cs, J = p.J;
+  const uint32_t rank = cluster_rank();
+  const int b = int(blockIdx.x / cs);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Tm = p.tr.T_max;
   const int64_t rb = int64_t(b) * Tm;
+  const int64_t S = int64_t(J) * SPEC_CHUNK;
+  const int64_t v0 = int64_t(rank) * S;
+  float *et = spec_dyn, *ed = spec_dyn + S;
+  const float k2 = p.k2;
+  // the root's rows towards L2 while the tree is checked
+  for (int j = 0; j < J; ++j) {
+    const int64_t e = v0 + int64_t(j) * SPEC_CHUNK + 8 * tid;
+    if (e < p.V) {
+      const char *tp = static_cast<const char *>(p.tgt) + (rb * p.row_stride + e) * int64_t(sizeof(T));
+      const char *dp = static_cast<const char *>(p.drf) + (rb * p.row_stride + e) * int64_t(sizeof(T));
+      asm volatile("prefetch.L2 [%0];" ::"l"(tp));
+      asm volatile("prefetch.L2 [%0];" ::"l"(dp));
+    }
+  }
   const int TL = __ldg(p.tr.tree_len + b), L = __ldg(p.tr.kv_len + b);
-  const int64_t V = p.tgt.V;
-  const int nseg = p.tgt.nseg;
-  const float k2 = p.tgt.k2;
-  // the tree's shape needs no statistics: checked while launch 1 runs
   if (warp == 0) {
     int bad = 0;
     if (TL < 1 || TL > Tm) {
@@ -1128,216 +1373,161 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       bad = ts.bad;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        s_par[lane + 32 * h] = ts.par[h];
-        s_tok[lane + 32 * h] = ts.tok[h];
+        sh.par[lane + 32 * h] = ts.par[h];
+        sh.tok[lane + 32 * h] = ts.tok[h];
       }
     }
     if (lane == 0) {
-      s_cmd[0] = bad;
-      if (bad) flag(p.status, bad);
+      sh.cmd = bad;
+      if (bad && rank == 0) flag(p.status, bad);
     }
   }
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   __syncthreads();
-  const int bad = s_cmd[0];
-  int n = -1, bonus = 0;
+  const bool bad = sh.cmd != 0;
+  int n = -1, bonus = 0, parity = 0;
   if (!bad) {
     int cur = 0;
     n = 0;
-    if (tid == 0) s_path[0] = 0;
+    if (tid == 0) sh.path[0] = 0;
     for (;;) {
       const int64_t row = rb + cur;
-      const T *trow = static_cast<const T *>(p.tgt.logits) + row * p.tgt.row_stride;
-      const T *drow = static_cast<const T *>(p.drf.logits) + row * p.drf.row_stride;
-      bool kids = false;
-      for (int c = cur + 1; c < TL && !kids; ++c) kids = s_par[c] == cur;
-      const bool try_kids = kids && n < p.max_path - 1;
-      if (warp == 0) {
-        const float2 mz = spec_row_mz(p.tgt.seg + row * nseg, nseg, k2);
-        if (lane == 0) s_rows[0] = mz.x, s_rows[1] = mz.y;
-      } else if (warp == 1 && try_kids) {
-        const float2 mz = spec_row_mz(p.drf.seg + row * nseg, nseg, k2);
-        if (lane == 0) s_rows[2] = mz.x, s_rows[3] = mz.y;
-      }
-      __syncthreads();
-      const float Mt = s_rows[0], Zt = s_rows[1], Md = s_rows[2], Zd = s_rows[3];
-      int k = 0, next = -1;
-      int eff = -1;  // the last rejection whose residual sum was positive (the draw's segment sums)
-      for (int c = cur + 1; c < TL && try_kids; ++c) {
-        if (s_par[c] != cur) continue;
-        if (tid == 0) {
-          const int x = s_tok[c];
-          float a = 0.f;
-          if (x >= 0 && x < V) {
-            const float pv = exp2f_approx((__uint_as_float(Elem<T>::bits(trow, x)) - Mt) * k2) / Zt;
-            const float qv = exp2f_approx((__uint_as_float(Elem<T>::bits(drow, x)) - Md) * k2) / Zd;
-            const float rv = spec_residual(pv, qv, s_zk, k);
-            a = qv > 0.f ? fminf(1.f, rv / qv) : (rv > 0.f ? 1.f : 0.f);
-          }
-          s_cmd[1] = __ldg(p.u_acc + rb + c) < a;
+      const T *trow = static_cast<const T *>(p.tgt) + row * p.row_stride;
+      const T *drow = static_cast<const T *>(p.drf) + row * p.row_stride;
+      // cur's children as a bit mask (nodes past tree_len hold parent -1)
+      const uint64_t kids = uint64_t(__ballot_sync(0xffffffffu, sh.par[lane] == cur && lane > cur)) |
+                            uint64_t(__ballot_sync(0xffffffffu, sh.par[lane + 32] == cur)) << 32;
+      const bool try_kids = kids != 0 && n < p.max_path - 1;
+      const bool mine_kid = tid < 64 && ((kids >> tid) & 1) && try_kids;
+      float kid_t = 0.f, kid_d = 0.f;  // the child's logits at its draft token (thread tid = child)
+      bool kid_in = false;
+      if (mine_kid) {
+        const int x = sh.tok[tid];
+        kid_in = x >= 0 && x < p.V;
+        if (kid_in) {
+          kid_t = __uint_as_float(Elem<T>::bits(trow, x));
+          kid_d = __uint_as_float(Elem<T>::bits(drow, x));
         }
-        __syncthreads();
-        if (s_cmd[1]) {
-          next = c;
+        sh.cu[tid] = __ldg(p.u_acc + rb + tid);
+      }
+      const float u_bonus = __ldg(p.u_res + rb + cur);
+      // the rows' maxima, then the exponentials and their sums
+      const float2 m = spec_load_rows<T>(p, trow, drow, try_kids, v0, et, ed);
+      spec_push<SpecMax>(sh, m, parity, cs, rank);
+      const float2 M = spec_combine<SpecMax>(sh, parity, cs);
+      parity ^= 1;
+      float2 z = make_float2(spec_exp_inplace(et, M.x, k2, J), 0.f);
+      if (try_kids) z.y = spec_exp_inplace(ed, M.y, k2, J);
+      if (mine_kid) {
+        sh.cet[tid] = kid_in ? exp2f_approx((kid_t - M.x) * k2) : 0.f;
+        sh.ced[tid] = kid_in ? exp2f_approx((kid_d - M.y) * k2) : 0.f;
+      }
+      spec_push<SpecSum>(sh, z, parity, cs, rank);
+      const float2 Z = spec_combine<SpecSum>(sh, parity, cs);
+      parity ^= 1;
+      const float Zd = Z.y;
+      float c = 0.f, Pu = Z.x;  // the residual ~ max(0, et - c ed), Pu its sum
+      int next = -1;
+      for (uint64_t rest = try_kids ? kids : 0; rest != 0; rest &= rest - 1) {
+        const int ch = __ffsll(static_cast<long long>(rest)) - 1;
+        const float et_x = sh.cet[ch], ed_x = sh.ced[ch];
+        const float num = fmaxf(fmaf(-c, ed_x, et_x), 0.f);
+        float a = 0.f;  // min(1, r(x) / q(x)) = Zd num / (Pu ed_x); q(x) = 0: 1 when r(x) > 0
+        if (num > 0.f) a = ed_x > 0.f ? fminf(1.f, (num / ed_x) * (Zd / Pu)) : 1.f;
+        if (sh.cu[ch] < a) {
+          next = ch;
           break;
         }
-        // a rejection: the residual's normaliser, and its sums per segment
-        // for a draw from it, in one pass over both rows. After a zero sum
-        // (r == q) the residual is kept, so every later sum at this node is
-        // zero too: no pass, and the sums of the last positive one stay.
-        const bool kept = k > 0 && s_zk[k - 1] == 0.f;
-        for (int g = warp; g < nseg && !kept; g += NW) {
-          float xt[4][8], xd[4][8];
+        // a rejection: the new residual's sum over the slice, then over the cluster
+        const float c2 = c + Pu / Zd;
+        float acc0 = 0.f, acc1 = 0.f;
+        for (int j = 0; j < J; ++j) {
+          const float4 *t4 = reinterpret_cast<const float4 *>(et + j * SPEC_CHUNK + 8 * tid);
+          const float4 *d4 = reinterpret_cast<const float4 *>(ed + j * SPEC_CHUNK + 8 * tid);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            sub_load<T>(trow, V, p.tgt.vec_ok, 4 * int64_t(g) + j, xt[j]);
-            sub_load<T>(drow, V, p.drf.vec_ok, 4 * int64_t(g) + j, xd[j]);
+          for (int h = 0; h < 2; ++h) {
+            const float4 tv = t4[h], dv = d4[h];
+            acc0 += spec_w(tv.x, dv.x, c2) + spec_w(tv.y, dv.y, c2);
+            acc1 += spec_w(tv.z, dv.z, c2) + spec_w(tv.w, dv.w, c2);
           }
-          float acc = 0.f;
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float pv = exp2f_approx((xt[j][e] - Mt) * k2) / Zt;
-              const float qv = exp2f_approx((xd[j][e] - Md) * k2) / Zd;
-              acc += fmaxf(spec_residual(pv, qv, s_zk, k) - qv, 0.f);
-            }
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-          if (lane == 0) s_seg[k & 1][g] = acc;
         }
-        __syncthreads();
-        if (warp == 0) {
-          float z = 0.f;
-          for (int g = lane; g < nseg && !kept; g += 32) z += s_seg[k & 1][g];
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
-          if (lane == 0) s_zk[k] = z;
-        }
-        __syncthreads();
-        // a zero sum (r == q) keeps the residual, and the sums it was drawn from
-        if (s_zk[k] > 0.f) eff = k;
-        ++k;
+        spec_push<SpecSum>(sh, make_float2(acc0 + acc1, 0.f), parity, cs, rank);
+        const float Pn = spec_combine<SpecSum>(sh, parity, cs).x;
+        parity ^= 1;
+        if (Pn > 0.f) c = c2, Pu = Pn;  // a zero sum (r == q) keeps the residual
       }
       if (next >= 0) {
         ++n;
         cur = next;
-        if (tid == 0) s_path[n] = next;
+        if (tid == 0) sh.path[n] = next;
         continue;
       }
-      // the bonus: a draw from the residual after k rejections (the target
-      // itself when k = 0) by inverse transform, one warp: segment weights in
-      // order up to the crossing, then the crossing segment's values
-      if (warp == 0) {
-        const float u0 = __ldg(p.u_res + rb + cur);
-        const float u = u0 > 0.f ? fminf(u0, 1.f) : 0.f;
-        auto seg_w = [&](int g) -> float {
-          if (g >= nseg) return 0.f;
-          if (eff < 0) {
-            const float2 v = __ldcg(p.tgt.seg + row * nseg + g);
-            return v.x == -INFINITY ? 0.f : v.y * exp2f_approx((v.x - Mt) * k2) / Zt;
-          }
-          return s_seg[eff & 1][g] / s_zk[eff];
-        };
-        int gs = -1, glast = -1;
-        float carry = 0.f, rem = 0.f;
-        for (int base = 0; base < nseg && gs < 0; base += 32) {
-          const float w = seg_w(base + lane);
-          float inc = w;
-#pragma unroll
-          for (int off = 1; off < 32; off <<= 1) {
-            const float y = __shfl_up_sync(0xffffffffu, inc, off);
-            if (lane >= off) inc += y;
-          }
-          const unsigned pos = __ballot_sync(0xffffffffu, w > 0.f);
-          if (pos) glast = base + 31 - __clz(pos);
-          const unsigned cross = __ballot_sync(0xffffffffu, w > 0.f && carry + inc > u);
-          if (cross) {
-            const int l0 = __ffs(cross) - 1;
-            gs = base + l0;
-            rem = u - (carry + __shfl_sync(0xffffffffu, inc - w, l0));
-          }
-          carry += __shfl_sync(0xffffffffu, inc, 31);
+      // the bonus: the weights max(0, et - c ed) (et when c = 0) per chunk,
+      // per slice and over the cluster; the slice where the running sum
+      // crosses u * total draws the entry
+      const bool use_q = c > 0.f;
+      float wj[SPEC_MAX_J];
+      int last;
+      const float tot = spec_weights(et, ed, c, use_q, J, wj, last);
+      spec_push<SpecSum>(sh, make_float2(tot, 0.f), parity, cs, rank);
+      // per-slice totals (lane r: slice r, its warps in order), then the
+      // crossing slice, the same on every warp of every CTA
+      float tr = 0.f;
+      if (lane < cs)
+        for (int w = 0; w < 16; ++w) tr += sh.slot[parity][lane * 16 + w].x;
+      parity ^= 1;
+      float total = 0.f;
+      for (int r = 0; r < cs; ++r) total += __shfl_sync(0xffffffffu, tr, r);
+      const float u = u_bonus > 0.f ? fminf(u_bonus, 1.f) : 0.f;
+      const float target = u * total;
+      int cr = -1, lastpos = -1;
+      float before = 0.f;
+      for (int r = 0; r < cs; ++r) {
+        const float t = __shfl_sync(0xffffffffu, tr, r);
+        if (t > 0.f) lastpos = r;
+        if (cr < 0) {
+          if (t > 0.f && before + t > target) cr = r;
+          else before += t;
         }
-        const bool tail = gs < 0;  // no crossing (u at the very end): the last value of positive weight
-        if (tail) gs = glast >= 0 ? glast : 0;
-        int pick = -1, lastpos = -1;
-        float acc = 0.f;
-        for (int j = 0; j < 4 && pick < 0; ++j) {
-          float xt[8], xd[8];
-          sub_load<T>(trow, V, p.tgt.vec_ok, 4 * int64_t(gs) + j, xt);
-          sub_load<T>(drow, V, p.drf.vec_ok, 4 * int64_t(gs) + j, xd);
-          float w[8], ls = 0.f;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float pv = exp2f_approx((xt[e] - Mt) * k2) / Zt;
-            w[e] = k == 0 ? pv : spec_residual(pv, exp2f_approx((xd[e] - Md) * k2) / Zd, s_zk, k);
-            ls += w[e];
-          }
-          float inc = ls;
-#pragma unroll
-          for (int off = 1; off < 32; off <<= 1) {
-            const float y = __shfl_up_sync(0xffffffffu, inc, off);
-            if (lane >= off) inc += y;
-          }
-          const int64_t e0 = int64_t(gs) * SEG + j * SUB + 8 * lane;
-          int lp = -1;
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (w[e] > 0.f) lp = int(e0) + e;
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, off));
-          if (lp >= 0) lastpos = lp;
-          if (!tail) {
-            const unsigned cross = __ballot_sync(0xffffffffu, acc + inc > rem && ls > 0.f);
-            if (cross) {
-              const int l0 = __ffs(cross) - 1;
-              int hit = -1;
-              if (lane == l0) {
-                float a = acc + inc - ls;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                  a += w[e];
-                  if (hit < 0 && w[e] > 0.f && a > rem) hit = int(e0) + e;
-                }
-                if (hit < 0) hit = lp;  // rounding: the last positive value of this lane's 8
-              }
-              pick = __shfl_sync(0xffffffffu, hit, l0);
-            }
-          }
-          acc += __shfl_sync(0xffffffffu, inc, 31);
-        }
-        if (pick < 0) pick = lastpos >= 0 ? lastpos : 0;
-        if (lane == 0) s_cmd[2] = int(std::min<int64_t>(std::max(pick, 0), V - 1));
       }
-      __syncthreads();
-      bonus = s_cmd[2];
+      const bool tail = cr < 0;
+      if (tail) cr = lastpos;
+      if (cr < 0) {  // no positive weight anywhere (rounding): token 0
+        if (rank == 0 && tid == 0) sh.bonus = 0;
+      } else if (int(rank) == cr) {
+        const int e = spec_slice_draw(sh, et, ed, c, use_q, wj, last, J, target - before, tail);
+        if (tid == 0) st_cluster_s32(&sh.bonus, 0, e >= 0 ? int32_t(v0 + e) : 0);
+      }
+      cluster_sync();
+      bonus = int(std::min<int64_t>(std::max(sh.bonus, 0), p.V - 1));  // used by rank 0 only
       break;
     }
   }
-  // outputs: path, drafts then the bonus, lengths (warp 0)
+  // outputs (rank 0): path, drafts then the bonus, lengths; the compaction is
+  // shared by the cluster's CTAs
   if (warp == 0) {
-    const int mp = p.max_path;
-    for (int kk = lane; kk < mp; kk += 32) {
-      int pv = -1, ov = -1;
-      if (n >= 0 && kk <= n) {
-        pv = s_path[kk];
-        ov = kk < n ? s_tok[s_path[kk + 1]] : bonus;
+    if (rank == 0) {
+      const int mp = p.max_path;
+      for (int kk = lane; kk < mp; kk += 32) {
+        int pv = -1, ov = -1;
+        if (n >= 0 && kk <= n) {
+          pv = sh.path[kk];
+          ov = kk < n ? sh.tok[sh.path[kk + 1]] : bonus;
+        }
+        p.path[int64_t(b) * mp + kk] = pv;
+        p.out_tokens[int64_t(b) * mp + kk] = ov;
       }
-      p.path[int64_t(b) * mp + kk] = pv;
-      p.out_tokens[int64_t(b) * mp + kk] = ov;
-    }
-    if (lane == 0) {
-      p.accept_len[b] = n >= 0 ? n + 1 : 0;
-      p.new_kv_len[b] = n >= 0 ? L + n + 1 : L;
+      if (lane == 0) {
+        p.accept_len[b] = n >= 0 ? n + 1 : 0;
+        p.new_kv_len[b] = n >= 0 ? L + n + 1 : L;
+      }
     }
     bool ok = n > 0;
-    if (ok) ok = move_offsets(p.kv, b, L, n, s_path, s_src, s_dst, p.status);
-    if (lane == 0) s_cmd[3] = ok ? n : 0;
+    if (ok) ok = move_offsets(p.kv, b, L, n, sh.path, sh.src, sh.dst, rank == 0 ? p.status : nullptr);
+    if (lane == 0) sh.cmd = ok ? n : 0;
   }
   __syncthreads();
-  const int nm = s_cmd[3];
-  if (nm > 0) compact_units(p.kv, nm, s_src, s_dst, tid, SPEC_THREADS);
+  const int nm = sh.cmd;
+  if (nm > 0) compact_units(p.kv, nm, sh.src, sh.dst, int64_t(rank) * SPEC_THREADS + tid, int64_t(cs) * SPEC_THREADS);
 }
 
 // ------------------------------------------------------------------ host side
@@ -1395,6 +1585,26 @@ dreams_status_t launch_dependent(void (*kernel)(Args...), dim3 grid, dim3 block,
     return DREAMS_ERR_CUDA;
   }
   return check_launch();
+}
+
+// CTAs per sequence of the speculative walk (a power of two): the fewest whose
+// slices of at most SPEC_MAX_J chunks cover V, doubled while every CTA keeps a
+// chunk of the vocabulary and the batch leaves SMs idle: up to 8, or 16 for
+// batches of at most 4 (clusters of 16 take most of a GPC each). cs = 0: V
+// too large.
+struct SpecPlan {
+  int cs, J;
+};
+inline SpecPlan plan_spec(int64_t B, int64_t V) {
+  const int64_t per_cta = int64_t(SPEC_MAX_J) * SPEC_CHUNK;
+  int cs = 1;
+  while (cs < SPEC_MAX_CS && int64_t(cs) * per_cta < V) cs *= 2;
+  if (int64_t(cs) * per_cta < V) return {0, 0};
+  const int64_t chunks = (V + SPEC_CHUNK - 1) / SPEC_CHUNK;
+  const int cap = B <= 4 ? 16 : 8;
+  while (cs < cap && B * cs * 2 <= num_sms() && chunks >= 2 * cs) cs *= 2;
+  const int64_t span = int64_t(cs) * SPEC_CHUNK;
+  return {cs, int((V + span - 1) / span)};
 }
 
 // Checks and fills the sampling parameters shared by both entry points.
@@ -1663,39 +1873,34 @@ extern "C" dreams_status_t dreams_verify_step_sampled(
   return launch_dependent(verify_tail_kernel, dim3(unsigned(tree->B)), dim3(TAIL_THREADS), s, p);
 }
 
-extern "C" size_t dreams_verify_step_speculative_workspace_size(const dreams_tree_t *tree, int64_t V) {
-  if (tree == nullptr || tree->B < 1 || tree->T_max < 1 || tree->T_max > 64 || V < 1) return 0;
-  const int64_t rows = int64_t(tree->B) * tree->T_max;
-  return 2 * sample_ws(rows, V);
-}
-
 extern "C" dreams_status_t dreams_verify_step_speculative(
     const void *target_logits, const void *draft_logits, dreams_dtype_t dtype, int64_t V, int64_t row_stride,
     const dreams_tree_t *tree, const dreams_kv_cache_t *kv, int32_t max_path, float temperature,
     const float *u_accept, const float *u_resample, int32_t *accept_len, int32_t *path, int32_t *out_tokens,
-    int32_t *new_kv_len, void *workspace, size_t workspace_bytes, int32_t *status_word, dreams_stream_t stream) {
+    int32_t *new_kv_len, int32_t *status_word, dreams_stream_t stream) {
   SpecParams p{};
   if (target_logits == nullptr || draft_logits == nullptr || u_accept == nullptr || u_resample == nullptr || V < 1 ||
-      V > INT_MAX - SEG || row_stride < V || !tree_params(tree, true, p.tr) || !kv_params(kv, p.kv) ||
-      max_path < 1 || max_path > 65 || accept_len == nullptr || path == nullptr || out_tokens == nullptr ||
-      new_kv_len == nullptr)
+      row_stride < V || !tree_params(tree, true, p.tr) || !kv_params(kv, p.kv) || max_path < 1 || max_path > 65 ||
+      accept_len == nullptr || path == nullptr || out_tokens == nullptr || new_kv_len == nullptr)
     return DREAMS_ERR_INVALID_ARG;
   if (dtype != DREAMS_F32 && dtype != DREAMS_BF16) return DREAMS_ERR_UNSUPPORTED;
   const size_t esz = dtype == DREAMS_F32 ? 4 : 2;
   if (reinterpret_cast<uintptr_t>(target_logits) % esz || reinterpret_cast<uintptr_t>(draft_logits) % esz ||
       (reinterpret_cast<uintptr_t>(u_accept) & 3) || (reinterpret_cast<uintptr_t>(u_resample) & 3))
     return DREAMS_ERR_INVALID_ARG;
-  if ((V + SEG - 1) / SEG > SPEC_MAX_SEG) return DREAMS_ERR_UNSUPPORTED;
-  const int64_t rows = int64_t(tree->B) * tree->T_max;
-  const size_t need = dreams_verify_step_speculative_workspace_size(tree, V);
-  if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace)) return DREAMS_ERR_WORKSPACE;
-  uint8_t *ws = static_cast<uint8_t *>(workspace);
-  int64_t ctas = 0, ctas_d = 0;
-  if (!sample_params(target_logits, dtype, rows, V, row_stride, temperature, u_resample, ws, p.tgt, ctas) ||
-      !sample_params(draft_logits, dtype, rows, V, row_stride, temperature, u_resample, ws + sample_ws(rows, V), p.drf,
-                     ctas_d))
-    return DREAMS_ERR_INVALID_ARG;
-  if (2 * ctas > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  const float k2 = 1.4426950408889634f / temperature;
+  if (!(temperature > 0.f) || !isfinite(temperature) || !isfinite(k2)) return DREAMS_ERR_INVALID_ARG;
+  const SpecPlan pl = plan_spec(tree->B, V);
+  if (pl.cs == 0) return DREAMS_ERR_UNSUPPORTED;
+  if (int64_t(tree->B) * pl.cs > INT_MAX) return DREAMS_ERR_UNSUPPORTED;
+  p.tgt = target_logits;
+  p.drf = draft_logits;
+  p.V = V;
+  p.row_stride = row_stride;
+  p.k2 = k2;
+  p.vec_ok = aligned16(target_logits) && aligned16(draft_logits) && (row_stride * int64_t(esz)) % 16 == 0;
+  p.cs = pl.cs;
+  p.J = pl.J;
   p.max_path = max_path;
   p.u_acc = u_accept;
   p.u_res = u_resample;
@@ -1704,15 +1909,36 @@ extern "C" dreams_status_t dreams_verify_step_speculative(
   p.out_tokens = out_tokens;
   p.new_kv_len = new_kv_len;
   p.status = status_word;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid(static_cast<unsigned>(2 * ctas));
-  if (dtype == DREAMS_F32) spec_stats_kernel<float><<<grid, SAMPLE_THREADS, 0, s>>>(p);
-  else spec_stats_kernel<__nv_bfloat16><<<grid, SAMPLE_THREADS, 0, s>>>(p);
-  const dreams_status_t st = check_launch();
+  const int smem = pl.J * SPEC_CHUNK * 2 * int(sizeof(float));
+  void (*kernel)(const SpecParams) =
+      dtype == DREAMS_F32 ? spec_walk_kernel<float> : spec_walk_kernel<__nv_bfloat16>;
+  dreams_status_t st = ensure_max_dynamic_smem(reinterpret_cast<const void *>(kernel), smem);
   if (st != DREAMS_OK) return st;
-  return dtype == DREAMS_F32
-             ? launch_dependent(spec_walk_kernel<float>, dim3(unsigned(tree->B)), dim3(SPEC_THREADS), s, p)
-             : launch_dependent(spec_walk_kernel<__nv_bfloat16>, dim3(unsigned(tree->B)), dim3(SPEC_THREADS), s, p);
+  if (pl.cs > 8) {
+    const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) {
+      set_last_cuda_error(e);
+      return DREAMS_ERR_CUDA;
+    }
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(int64_t(tree->B) * pl.cs));
+  cfg.blockDim = dim3(SPEC_THREADS);
+  cfg.dynamicSmemBytes = size_t(smem);
+  cfg.stream = reinterpret_cast<cudaStream_t>(stream);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = unsigned(pl.cs);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, p);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return DREAMS_ERR_CUDA;
+  }
+  return check_launch();
 }
 
 // ------------------------------------------------------------------ no-allocation argmax

@@ -164,13 +164,9 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert vs(P, 3, 1000, 1000, ctypes.byref(tr), ctypes.byref(kvc), 5, null, P, P, P, P, P, wsb, st,
               s) == dreams.ERR_UNSUPPORTED
 
-    wss = lib.dreams_verify_step_speculative_workspace_size(ctypes.byref(tr), 1000)
-    assert wss > 0 and wss % 16 == 0
-    assert lib.dreams_verify_step_speculative_workspace_size(ctypes.byref(tr), 0) == 0
-
-    def spec(tgt=P, drf=P, dt=1, V=1000, rs=1000, tree=tr, mp=5, tau=1.0, ua=P, ur=P, ws=P, wsb=wss):
+    def spec(tgt=P, drf=P, dt=1, V=1000, rs=1000, tree=tr, mp=5, tau=1.0, ua=P, ur=P):
         return lib.dreams_verify_step_speculative(tgt, drf, dt, V, rs, ctypes.byref(tree), ctypes.byref(kvc), mp,
-                                                  tau, ua, ur, P, P, P, P, ws, wsb, st, s)
+                                                  tau, ua, ur, P, P, P, P, st, s)
 
     assert spec(tgt=null) == dreams.ERR_INVALID_ARG
     assert spec(drf=null) == dreams.ERR_INVALID_ARG
@@ -182,11 +178,10 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert spec(mp=66) == dreams.ERR_INVALID_ARG
     assert spec(tree=dreams._Tree(P, null, P, P, 2, 8)) == dreams.ERR_INVALID_ARG  # the drafts are needed
     assert spec(dt=7) == dreams.ERR_UNSUPPORTED
-    assert spec(V=524289, rs=524289) == dreams.ERR_UNSUPPORTED  # beyond the walk's per-segment sums
-    assert spec(wsb=wss - 1) == dreams.ERR_WORKSPACE
-    assert spec(ws=P + 8) == dreams.ERR_WORKSPACE
+    assert spec(V=393217, rs=393217) == dreams.ERR_UNSUPPORTED  # more than 16 CTAs' shared memory
     assert spec(tau=0.0) == dreams.ERR_INVALID_ARG
     assert spec(tau=float("nan")) == dreams.ERR_INVALID_ARG
+    assert spec(tau=1e-45) == dreams.ERR_INVALID_ARG         # log2(e) / tau overflows
 
 
 def test_stall_hook_argument_checks(lib):

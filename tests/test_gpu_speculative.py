@@ -285,9 +285,9 @@ def test_malformed_tree_is_flagged(dreams):
             np.testing.assert_array_equal(r[key][b].cpu().numpy(), ref[key][b], err_msg=key)
 
 
-def test_speculative_repeatable_and_workspace_free_of_state(dreams):
-    """Two calls on one workspace, with garbage written into it between them,
-    give identical outputs: the workspace carries no state."""
+def test_speculative_repeatable(dreams):
+    """Two calls on the same inputs give identical outputs (the sums are
+    combined in a fixed order, whichever SM ran each CTA)."""
     w = W.make("qwen2vl7b", with_attn=False)
     rng = np.random.default_rng(3)
     drf = (w.logits.float() + torch.from_numpy(0.4 * rng.standard_normal(w.logits.shape).astype(np.float32))).to(
@@ -297,14 +297,11 @@ def test_speculative_repeatable_and_workspace_free_of_state(dreams):
     k = torch.zeros((w.B, cap, 1, 8), dtype=torch.bfloat16, device="cuda")
     kv = dreams.KVCache(k, k.clone())
     tree = dreams.Tree(w.parent.cuda(), w.tokens.cuda(), w.tree_len.cuda(), w.kv_len.cuda())
-    need = dreams.verify_step_speculative_workspace_size(tree, w.V)
-    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
     u_acc = torch.from_numpy(rng.random((w.B, w.T_max), dtype=np.float32)).cuda()
     u_res = torch.from_numpy(rng.random((w.B, w.T_max), dtype=np.float32)).cuda()
-    a = dreams.verify_step_speculative(tgt, drf, tree, kv, w.max_path, 1.0, u_acc, u_res, workspace=ws)
+    a = dreams.verify_step_speculative(tgt, drf, tree, kv, w.max_path, 1.0, u_acc, u_res)
     a = {key: t.clone() for key, t in a.items()}
-    ws.fill_(0x7F)
-    b = dreams.verify_step_speculative(tgt, drf, tree, kv, w.max_path, 1.0, u_acc, u_res, workspace=ws)
+    b = dreams.verify_step_speculative(tgt, drf, tree, kv, w.max_path, 1.0, u_acc, u_res)
     torch.cuda.synchronize()
     for key in a:
         assert torch.equal(a[key], b[key]), key
