@@ -1036,12 +1036,15 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
 //
 // One thread-block cluster per sequence; CTA `rank` of the cluster holds the
 // vocabulary slice [rank * S, (rank + 1) * S) of the rows of the node being
-// visited, as exponentials in shared memory. Only the rows of visited nodes
-// are read. A sum (or maximum) over the vocabulary: every warp reduces its
-// threads' values and stores the result into every CTA's shared memory
-// (distributed shared memory), one cluster barrier, then each warp combines
-// the cs * 16 values in the same fixed order: all CTAs hold bit-identical
-// results, take the same decisions and pass the same cluster barriers.
+// visited, as exponentials in shared memory (each thread's relative to its own
+// maximum m, with the factor a = 2^((m - M) k2) to the row's maximum M kept in
+// a register). Only the rows of visited nodes are read. A sum over the
+// vocabulary: every warp reduces its threads' values and stores the result
+// into every CTA's shared memory (distributed shared memory), one cluster
+// barrier, then each warp combines the cs * 16 values in the same fixed order:
+// all CTAs hold bit-identical results, take the same decisions and pass the
+// same cluster barriers. A row's (M, Zt) and the draft's (M, Zd) take one such
+// exchange of per-warp (maximum, sum) pairs.
 constexpr int SPEC_THREADS = 512;                    // 16 warps
 constexpr int SPEC_CHUNK = 8 * SPEC_THREADS;         // values per chunk: 8 per thread
 constexpr int SPEC_MAX_J = 6;                        // chunks per CTA slice (192 KB of f32 pairs)
@@ -1080,8 +1083,9 @@ __device__ __forceinline__ uint32_t cluster_addr(const void *local_ptr, uint32_t
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
   return ra;
 }
-__device__ __forceinline__ void st_cluster_f2(const float2 *local_ptr, uint32_t rank, float2 v) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(cluster_addr(local_ptr, rank)), "f"(v.x), "f"(v.y)
+__device__ __forceinline__ void st_cluster_f4(const float4 *local_ptr, uint32_t rank, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(cluster_addr(local_ptr, rank)), "f"(v.x),
+               "f"(v.y), "f"(v.z), "f"(v.w)
                : "memory");
 }
 __device__ __forceinline__ void st_cluster_s32(const int32_t *local_ptr, uint32_t rank, int32_t v) {
@@ -1089,63 +1093,92 @@ __device__ __forceinline__ void st_cluster_s32(const int32_t *local_ptr, uint32_
 }
 
 struct SpecShared {
-  float2 slot[2][SPEC_MAX_CS * 16];  // [parity][rank * 16 + warp]: every warp's partial of every CTA
+  float4 slot[2][SPEC_MAX_CS * 16];  // [parity][rank * 16 + warp]: every warp's partial of every CTA
   float chunk[SPEC_MAX_J][16];       // the bonus draw: per-warp sums of each chunk
   int32_t hit[16], last[16];
   int32_t par[64], tok[64], path[65];
   int64_t src[65], dst[65];
-  float cet[64], ced[64];  // exponentials of the target / draft logits at each child's draft token
+  float cxt[64], cxd[64];  // the target / draft logits at each child's draft token
   float cu[64];            // u_acc of each child
   int32_t pick;            // the draw inside this CTA's slice
   int32_t bonus;           // rank 0: the bonus token, written by the CTA that drew it
   int32_t cmd;
 };
 
-struct SpecMax {
-  __device__ static float f(float a, float b) { return fmaxf(a, b); }
-  __device__ static float id() { return -INFINITY; }
-};
-struct SpecSum {
-  __device__ static float f(float a, float b) { return a + b; }
-  __device__ static float id() { return 0.f; }
-};
-
-// Each warp reduces its threads' pairs and stores the result into slot
-// [parity][rank * 16 + warp] of every CTA of the cluster; then the cluster
-// barrier. No thread reads another CTA's memory afterwards.
-template <class Op>
-__device__ __forceinline__ void spec_push(SpecShared &sh, float2 v, int parity, int cs, uint32_t rank) {
+// Stores a warp-uniform value into slot [parity][rank * 16 + warp] of every
+// CTA of the cluster, then the cluster barrier. No thread reads another CTA's
+// memory afterwards.
+__device__ __forceinline__ void spec_push(SpecShared &sh, float4 v, int parity, int cs, uint32_t rank) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    v.x = Op::f(v.x, __shfl_xor_sync(0xffffffffu, v.x, off));
-    v.y = Op::f(v.y, __shfl_xor_sync(0xffffffffu, v.y, off));
-  }
-  v.x = __shfl_sync(0xffffffffu, v.x, 0);  // lane 0's bits on every lane
-  v.y = __shfl_sync(0xffffffffu, v.y, 0);
-  if (lane < cs) st_cluster_f2(&sh.slot[parity][rank * 16 + warp], uint32_t(lane), v);
+  if (lane < cs) st_cluster_f4(&sh.slot[parity][rank * 16 + warp], uint32_t(lane), v);
   cluster_sync();
 }
 
-// The combination of all cs * 16 pushed pairs in the same fixed order in every
-// warp of every CTA, so the bits agree everywhere.
-template <class Op>
-__device__ __forceinline__ float2 spec_combine(const SpecShared &sh, int parity, int cs) {
+__device__ __forceinline__ float warp_sum_bcast(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return __shfl_sync(0xffffffffu, v, 0);  // lane 0's bits on every lane
+}
+
+// A sum over the cluster: the warps' sums pushed, then combined in the same
+// fixed order in every warp of every CTA (so the bits agree everywhere).
+__device__ __forceinline__ float spec_cluster_sum(SpecShared &sh, float v, int parity, int cs, uint32_t rank) {
+  spec_push(sh, make_float4(warp_sum_bcast(v), 0.f, 0.f, 0.f), parity, cs, rank);
+  float acc = 0.f;
+  for (int i = threadIdx.x & 31; i < cs * 16; i += 32) acc += sh.slot[parity][i].x;
+  return warp_sum_bcast(acc);
+}
+
+// The rows' maxima and exponential sums over the cluster from each thread's
+// (m_t, s_t, m_d, s_d), s = sum 2^((x - m) k2): (Mt, Zt, Md, Zd). Per warp the
+// maxima, then the sums rescaled to them; across the cluster the same.
+__device__ float4 spec_cluster_ms(SpecShared &sh, float4 v, int parity, int cs, uint32_t rank, float k2) {
+  float Mt = v.x, Md = v.z;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, off));
+    Md = fmaxf(Md, __shfl_xor_sync(0xffffffffu, Md, off));
+  }
+  const float st = v.x == -INFINITY ? 0.f : v.y * exp2f_approx((v.x - Mt) * k2);
+  const float sd = v.z == -INFINITY ? 0.f : v.w * exp2f_approx((v.z - Md) * k2);
+  spec_push(sh, make_float4(Mt, warp_sum_bcast(st), Md, warp_sum_bcast(sd)), parity, cs, rank);
   const int lane = threadIdx.x & 31;
-  float2 acc = make_float2(Op::id(), Op::id());
+  float mt = -INFINITY, md = -INFINITY;
   for (int i = lane; i < cs * 16; i += 32) {
-    const float2 v = sh.slot[parity][i];
-    acc.x = Op::f(acc.x, v.x);
-    acc.y = Op::f(acc.y, v.y);
+    mt = fmaxf(mt, sh.slot[parity][i].x);
+    md = fmaxf(md, sh.slot[parity][i].z);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    acc.x = Op::f(acc.x, __shfl_xor_sync(0xffffffffu, acc.x, off));
-    acc.y = Op::f(acc.y, __shfl_xor_sync(0xffffffffu, acc.y, off));
+    mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, off));
+    md = fmaxf(md, __shfl_xor_sync(0xffffffffu, md, off));
   }
-  acc.x = __shfl_sync(0xffffffffu, acc.x, 0);
-  acc.y = __shfl_sync(0xffffffffu, acc.y, 0);
-  return acc;
+  float zt = 0.f, zd = 0.f;
+  for (int i = lane; i < cs * 16; i += 32) {
+    const float4 e = sh.slot[parity][i];
+    if (e.x != -INFINITY) zt += e.y * exp2f_approx((e.x - mt) * k2);
+    if (e.z != -INFINITY) zd += e.w * exp2f_approx((e.z - md) * k2);
+  }
+  return make_float4(mt, warp_sum_bcast(zt), md, warp_sum_bcast(zd));
+}
+
+// Warp 0: the parent and token rows of a sequence into sh (entries past
+// tree_len: parent -1, token 0); DREAMS_DATA_BAD_PARENT when parent[0] != -1
+// or a parent[i] lies outside [0, i).
+__device__ int spec_tree_warp(SpecShared &sh, const int32_t *par_row, const int32_t *tok_row, int T) {
+  const int lane = threadIdx.x & 31;
+  int bad = 0;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i = lane + 32 * h;
+    const bool live = i < T;
+    const int pa = live ? __ldg(par_row + i) : -1;
+    sh.par[i] = pa;
+    sh.tok[i] = live ? __ldg(tok_row + i) : 0;
+    if (i == 0) bad |= pa != -1;
+    else if (live) bad |= pa < 0 || pa >= i;
+  }
+  return __any_sync(0xffffffffu, bad) ? DREAMS_DATA_BAD_PARENT : 0;
 }
 
 // This thread's values of one slice as floats into e (values past V: -inf);
@@ -1206,8 +1239,16 @@ __device__ float2 spec_load_rows(const SpecParams &p, const T *trow, const T *dr
 }
 
 // e <- 2^((e - M) k2) in place over this thread's values; returns their sum.
+// M = -inf (every value past V): zeros.
 __device__ __forceinline__ float spec_exp_inplace(float *e, float M, float k2, int J) {
   const int tid = threadIdx.x;
+  if (M == -INFINITY) {
+    for (int j = 0; j < J; ++j) {
+      float4 *q = reinterpret_cast<float4 *>(e + j * SPEC_CHUNK + 8 * tid);
+      q[0] = q[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    return 0.f;
+  }
   float s0 = 0.f, s1 = 0.f;
   for (int j = 0; j < J; ++j) {
     float4 *q = reinterpret_cast<float4 *>(e + j * SPEC_CHUNK + 8 * tid);
@@ -1229,9 +1270,10 @@ __device__ __forceinline__ float spec_exp_inplace(float *e, float M, float k2, i
 // The residual's numerator at one vocabulary entry: max(0, et - c ed).
 __device__ __forceinline__ float spec_w(float et, float ed, float c) { return fmaxf(fmaf(-c, ed, et), 0.f); }
 
-// Sum of the residual's numerator over this thread's values (et alone when
-// use_q is false); per chunk into wj, and the last index of positive weight.
-__device__ __forceinline__ float spec_weights(const float *et, const float *ed, float c, bool use_q, int J,
+// The residual's numerator over this thread's values, a_t max(0, et - ct ed)
+// (a_t et alone when use_q is false): its sum, per chunk into wj, and the last
+// index of positive weight.
+__device__ __forceinline__ float spec_weights(const float *et, const float *ed, float at, float ct, bool use_q, int J,
                                               float (&wj)[SPEC_MAX_J], int &last) {
   const int tid = threadIdx.x;
   float tot = 0.f;
@@ -1249,14 +1291,15 @@ __device__ __forceinline__ float spec_weights(const float *et, const float *ed, 
         const float4 tv = t4[h];
         if (use_q) {
           const float4 dv = d4[h];
-          w[4 * h] = spec_w(tv.x, dv.x, c), w[4 * h + 1] = spec_w(tv.y, dv.y, c);
-          w[4 * h + 2] = spec_w(tv.z, dv.z, c), w[4 * h + 3] = spec_w(tv.w, dv.w, c);
+          w[4 * h] = spec_w(tv.x, dv.x, ct), w[4 * h + 1] = spec_w(tv.y, dv.y, ct);
+          w[4 * h + 2] = spec_w(tv.z, dv.z, ct), w[4 * h + 3] = spec_w(tv.w, dv.w, ct);
         } else {
           w[4 * h] = tv.x, w[4 * h + 1] = tv.y, w[4 * h + 2] = tv.z, w[4 * h + 3] = tv.w;
         }
       }
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
+        w[i] *= at;
         wj[j] += w[i];
         if (w[i] > 0.f) last = e0 + i;
       }
@@ -1270,7 +1313,7 @@ __device__ __forceinline__ float spec_weights(const float *et, const float *ed, 
 // the weights (in vocabulary order) first exceeds rem; tail: the last entry
 // of positive weight. Returns the slice-relative index (-1: no positive
 // weight) on every thread of the CTA.
-__device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed, float c, bool use_q,
+__device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed, float at, float ct, bool use_q,
                                const float (&wj)[SPEC_MAX_J], int last, int J, float rem, bool tail) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 #pragma unroll
@@ -1324,7 +1367,7 @@ __device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed,
     float a = excl;
     int hit = -1, lp = -1;
     for (int i = 0; i < 8; ++i) {
-      const float w = use_q ? spec_w(et[e0 + i], ed[e0 + i], c) : et[e0 + i];
+      const float w = at * (use_q ? spec_w(et[e0 + i], ed[e0 + i], ct) : et[e0 + i]);
       a += w;
       if (w > 0.f) lp = e0 + i;
       if (hit < 0 && w > 0.f && a > rem) hit = e0 + i;
@@ -1364,19 +1407,9 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
   const int TL = __ldg(p.tr.tree_len + b), L = __ldg(p.tr.kv_len + b);
   if (warp == 0) {
     int bad = 0;
-    if (TL < 1 || TL > Tm) {
-      bad = DREAMS_DATA_BAD_TREE_LEN;
-    } else if (L < 0 || L > p.kv.capacity - TL) {
-      bad = DREAMS_DATA_BAD_KV_LEN;
-    } else {
-      const TreeShape ts = tree_shape_warp(p.tr.parent + rb, p.tr.tokens + rb, TL);
-      bad = ts.bad;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        sh.par[lane + 32 * h] = ts.par[h];
-        sh.tok[lane + 32 * h] = ts.tok[h];
-      }
-    }
+    if (TL < 1 || TL > Tm) bad = DREAMS_DATA_BAD_TREE_LEN;
+    else if (L < 0 || L > p.kv.capacity - TL) bad = DREAMS_DATA_BAD_KV_LEN;
+    else bad = spec_tree_warp(sh, p.tr.parent + rb, p.tr.tokens + rb, TL);
     if (lane == 0) {
       sh.cmd = bad;
       if (bad && rank == 0) flag(p.status, bad);
@@ -1397,39 +1430,33 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       const uint64_t kids = uint64_t(__ballot_sync(0xffffffffu, sh.par[lane] == cur && lane > cur)) |
                             uint64_t(__ballot_sync(0xffffffffu, sh.par[lane + 32] == cur)) << 32;
       const bool try_kids = kids != 0 && n < p.max_path - 1;
-      const bool mine_kid = tid < 64 && ((kids >> tid) & 1) && try_kids;
-      float kid_t = 0.f, kid_d = 0.f;  // the child's logits at its draft token (thread tid = child)
-      bool kid_in = false;
-      if (mine_kid) {
+      // each child's logits at its draft token and its uniform, loaded while
+      // the rows are (children have larger indices than every node read before)
+      if (try_kids && tid < 64 && ((kids >> tid) & 1)) {
         const int x = sh.tok[tid];
-        kid_in = x >= 0 && x < p.V;
-        if (kid_in) {
-          kid_t = __uint_as_float(Elem<T>::bits(trow, x));
-          kid_d = __uint_as_float(Elem<T>::bits(drow, x));
-        }
+        const bool in = x >= 0 && x < p.V;
+        sh.cxt[tid] = in ? __uint_as_float(Elem<T>::bits(trow, x)) : -INFINITY;
+        sh.cxd[tid] = in ? __uint_as_float(Elem<T>::bits(drow, x)) : -INFINITY;
         sh.cu[tid] = __ldg(p.u_acc + rb + tid);
       }
       const float u_bonus = __ldg(p.u_res + rb + cur);
-      // the rows' maxima, then the exponentials and their sums
+      // the rows' maxima and exponential sums: per thread, then over the cluster
       const float2 m = spec_load_rows<T>(p, trow, drow, try_kids, v0, et, ed);
-      spec_push<SpecMax>(sh, m, parity, cs, rank);
-      const float2 M = spec_combine<SpecMax>(sh, parity, cs);
+      const float st = spec_exp_inplace(et, m.x, k2, J);
+      const float sd = try_kids ? spec_exp_inplace(ed, m.y, k2, J) : 0.f;
+      const float4 g = spec_cluster_ms(sh, make_float4(m.x, st, m.y, sd), parity, cs, rank, k2);
       parity ^= 1;
-      float2 z = make_float2(spec_exp_inplace(et, M.x, k2, J), 0.f);
-      if (try_kids) z.y = spec_exp_inplace(ed, M.y, k2, J);
-      if (mine_kid) {
-        sh.cet[tid] = kid_in ? exp2f_approx((kid_t - M.x) * k2) : 0.f;
-        sh.ced[tid] = kid_in ? exp2f_approx((kid_d - M.y) * k2) : 0.f;
-      }
-      spec_push<SpecSum>(sh, z, parity, cs, rank);
-      const float2 Z = spec_combine<SpecSum>(sh, parity, cs);
-      parity ^= 1;
-      const float Zd = Z.y;
-      float c = 0.f, Pu = Z.x;  // the residual ~ max(0, et - c ed), Pu its sum
+      const float Mt = g.x, Zd = g.w;
+      // this thread's factors to the rows' maxima (its exponentials are
+      // relative to its own maxima), and their ratio for the passes
+      const float at = m.x == -INFINITY ? 0.f : exp2f_approx((m.x - Mt) * k2);
+      const float ad = m.y == -INFINITY ? 0.f : exp2f_approx((m.y - g.z) * k2);
+      const float rd = at > 0.f ? ad / at : 0.f;
+      float c = 0.f, Pu = g.y;  // the residual ~ max(0, et - c ed), Pu its sum
       int next = -1;
       for (uint64_t rest = try_kids ? kids : 0; rest != 0; rest &= rest - 1) {
         const int ch = __ffsll(static_cast<long long>(rest)) - 1;
-        const float et_x = sh.cet[ch], ed_x = sh.ced[ch];
+        const float et_x = exp2f_approx((sh.cxt[ch] - Mt) * k2), ed_x = exp2f_approx((sh.cxd[ch] - g.z) * k2);
         const float num = fmaxf(fmaf(-c, ed_x, et_x), 0.f);
         float a = 0.f;  // min(1, r(x) / q(x)) = Zd num / (Pu ed_x); q(x) = 0: 1 when r(x) > 0
         if (num > 0.f) a = ed_x > 0.f ? fminf(1.f, (num / ed_x) * (Zd / Pu)) : 1.f;
@@ -1438,20 +1465,19 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
           break;
         }
         // a rejection: the new residual's sum over the slice, then over the cluster
-        const float c2 = c + Pu / Zd;
+        const float c2 = c + Pu / Zd, ct = c2 * rd;
         float acc0 = 0.f, acc1 = 0.f;
-        for (int j = 0; j < J; ++j) {
+        for (int j = 0; j < J && at > 0.f; ++j) {
           const float4 *t4 = reinterpret_cast<const float4 *>(et + j * SPEC_CHUNK + 8 * tid);
           const float4 *d4 = reinterpret_cast<const float4 *>(ed + j * SPEC_CHUNK + 8 * tid);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const float4 tv = t4[h], dv = d4[h];
-            acc0 += spec_w(tv.x, dv.x, c2) + spec_w(tv.y, dv.y, c2);
-            acc1 += spec_w(tv.z, dv.z, c2) + spec_w(tv.w, dv.w, c2);
+            acc0 += spec_w(tv.x, dv.x, ct) + spec_w(tv.y, dv.y, ct);
+            acc1 += spec_w(tv.z, dv.z, ct) + spec_w(tv.w, dv.w, ct);
           }
         }
-        spec_push<SpecSum>(sh, make_float2(acc0 + acc1, 0.f), parity, cs, rank);
-        const float Pn = spec_combine<SpecSum>(sh, parity, cs).x;
+        const float Pn = spec_cluster_sum(sh, at * (acc0 + acc1), parity, cs, rank);
         parity ^= 1;
         if (Pn > 0.f) c = c2, Pu = Pn;  // a zero sum (r == q) keeps the residual
       }
@@ -1465,10 +1491,11 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       // per slice and over the cluster; the slice where the running sum
       // crosses u * total draws the entry
       const bool use_q = c > 0.f;
+      const float ct = c * rd;
       float wj[SPEC_MAX_J];
       int last;
-      const float tot = spec_weights(et, ed, c, use_q, J, wj, last);
-      spec_push<SpecSum>(sh, make_float2(tot, 0.f), parity, cs, rank);
+      const float tot = spec_weights(et, ed, at, ct, use_q, J, wj, last);
+      spec_push(sh, make_float4(warp_sum_bcast(tot), 0.f, 0.f, 0.f), parity, cs, rank);
       // per-slice totals (lane r: slice r, its warps in order), then the
       // crossing slice, the same on every warp of every CTA
       float tr = 0.f;
@@ -1494,7 +1521,7 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       if (cr < 0) {  // no positive weight anywhere (rounding): token 0
         if (rank == 0 && tid == 0) sh.bonus = 0;
       } else if (int(rank) == cr) {
-        const int e = spec_slice_draw(sh, et, ed, c, use_q, wj, last, J, target - before, tail);
+        const int e = spec_slice_draw(sh, et, ed, at, ct, use_q, wj, last, J, target - before, tail);
         if (tid == 0) st_cluster_s32(&sh.bonus, 0, e >= 0 ? int32_t(v0 + e) : 0);
       }
       cluster_sync();
