@@ -1039,12 +1039,12 @@ __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepPar
 // visited, as exponentials in shared memory (each thread's relative to its own
 // maximum m, with the factor a = 2^((m - M) k2) to the row's maximum M kept in
 // a register). Only the rows of visited nodes are read. A sum over the
-// vocabulary: every warp reduces its threads' values and stores the result
-// into every CTA's shared memory (distributed shared memory), one cluster
-// barrier, then each warp combines the cs * 16 values in the same fixed order:
+// vocabulary: warps reduce their threads' values, warp 0 the warps' and stores
+// the CTA's value into every CTA's shared memory (distributed shared memory),
+// one cluster barrier, then each warp combines the cs values in rank order:
 // all CTAs hold bit-identical results, take the same decisions and pass the
-// same cluster barriers. A row's (M, Zt) and the draft's (M, Zd) take one such
-// exchange of per-warp (maximum, sum) pairs.
+// same cluster barriers. The rows' maxima and exponential sums take one such
+// exchange of (maximum, sum) pairs.
 constexpr int SPEC_THREADS = 512;                    // 16 warps
 constexpr int SPEC_CHUNK = 8 * SPEC_THREADS;         // values per chunk: 8 per thread
 constexpr int SPEC_MAX_J = 6;                        // chunks per CTA slice (192 KB of f32 pairs)
@@ -1093,8 +1093,10 @@ __device__ __forceinline__ void st_cluster_s32(const int32_t *local_ptr, uint32_
 }
 
 struct SpecShared {
-  float4 slot[2][SPEC_MAX_CS * 16];  // [parity][rank * 16 + warp]: every warp's partial of every CTA
+  float4 slot[2][SPEC_MAX_CS];       // [parity][rank]: every CTA's partial of the current exchange
   float chunk[SPEC_MAX_J][16];       // the bonus draw: per-warp sums of each chunk
+  float red[16];                     // the bonus draw: per-warp sums of the slice
+  float4 red4[16];                   // per-warp partials of a sum or of (maximum, sum) pairs
   int32_t hit[16], last[16];
   int32_t par[64], tok[64], path[65];
   int64_t src[65], dst[65];
@@ -1105,13 +1107,29 @@ struct SpecShared {
   int32_t cmd;
 };
 
-// Stores a warp-uniform value into slot [parity][rank * 16 + warp] of every
-// CTA of the cluster, then the cluster barrier. No thread reads another CTA's
-// memory afterwards.
-__device__ __forceinline__ void spec_push(SpecShared &sh, float4 v, int parity, int cs, uint32_t rank) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane < cs) st_cluster_f4(&sh.slot[parity][rank * 16 + warp], uint32_t(lane), v);
-  cluster_sync();
+// Loads issued where they stand (volatile), so that their latency overlaps the
+// work between the load and the first use of its value.
+__device__ __forceinline__ int ld_issue_now(const int32_t *ptr) {
+  int v;
+  asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(ptr));
+  return v;
+}
+__device__ __forceinline__ float ld_now_f32(const float *ptr) {
+  float v;
+  asm volatile("ld.global.nc.f32 %0, [%1];" : "=f"(v) : "l"(ptr));
+  return v;
+}
+template <typename T>
+__device__ __forceinline__ float ld_now_val(const T *ptr);
+template <>
+__device__ __forceinline__ float ld_now_val<float>(const float *ptr) {
+  return ld_now_f32(ptr);
+}
+template <>
+__device__ __forceinline__ float ld_now_val<__nv_bfloat16>(const __nv_bfloat16 *ptr) {
+  unsigned short v;
+  asm volatile("ld.global.nc.u16 %0, [%1];" : "=h"(v) : "l"(ptr));
+  return __uint_as_float(uint32_t(v) << 16);
 }
 
 __device__ __forceinline__ float warp_sum_bcast(float v) {
@@ -1120,19 +1138,9 @@ __device__ __forceinline__ float warp_sum_bcast(float v) {
   return __shfl_sync(0xffffffffu, v, 0);  // lane 0's bits on every lane
 }
 
-// A sum over the cluster: the warps' sums pushed, then combined in the same
-// fixed order in every warp of every CTA (so the bits agree everywhere).
-__device__ __forceinline__ float spec_cluster_sum(SpecShared &sh, float v, int parity, int cs, uint32_t rank) {
-  spec_push(sh, make_float4(warp_sum_bcast(v), 0.f, 0.f, 0.f), parity, cs, rank);
-  float acc = 0.f;
-  for (int i = threadIdx.x & 31; i < cs * 16; i += 32) acc += sh.slot[parity][i].x;
-  return warp_sum_bcast(acc);
-}
-
-// The rows' maxima and exponential sums over the cluster from each thread's
-// (m_t, s_t, m_d, s_d), s = sum 2^((x - m) k2): (Mt, Zt, Md, Zd). Per warp the
-// maxima, then the sums rescaled to them; across the cluster the same.
-__device__ float4 spec_cluster_ms(SpecShared &sh, float4 v, int parity, int cs, uint32_t rank, float k2) {
+// (maximum, sum of 2^((x - maximum) k2)) of two rows over the warp's lanes,
+// from each lane's pair (x, y) and (z, w); lane 0's bits on every lane.
+__device__ __forceinline__ float4 ms4_lanes(float4 v, float k2) {
   float Mt = v.x, Md = v.z;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -1141,40 +1149,55 @@ __device__ float4 spec_cluster_ms(SpecShared &sh, float4 v, int parity, int cs, 
   }
   const float st = v.x == -INFINITY ? 0.f : v.y * exp2f_approx((v.x - Mt) * k2);
   const float sd = v.z == -INFINITY ? 0.f : v.w * exp2f_approx((v.z - Md) * k2);
-  spec_push(sh, make_float4(Mt, warp_sum_bcast(st), Md, warp_sum_bcast(sd)), parity, cs, rank);
-  const int lane = threadIdx.x & 31;
-  float mt = -INFINITY, md = -INFINITY;
-  for (int i = lane; i < cs * 16; i += 32) {
-    mt = fmaxf(mt, sh.slot[parity][i].x);
-    md = fmaxf(md, sh.slot[parity][i].z);
+  return make_float4(Mt, warp_sum_bcast(st), Md, warp_sum_bcast(sd));
+}
+
+// A sum over the cluster: warps, then warp 0 over the warps, then one value
+// per CTA into slot [parity][rank] of every CTA; after the cluster barrier
+// every warp combines the cs values in lane order (the same bits everywhere).
+__device__ __forceinline__ float spec_cluster_sum(SpecShared &sh, float v, int parity, int cs, uint32_t rank) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float wv = warp_sum_bcast(v);
+  if (lane == 0) sh.red4[warp] = make_float4(wv, 0.f, 0.f, 0.f);
+  __syncthreads();
+  if (warp == 0) {
+    const float cta = warp_sum_bcast(lane < 16 ? sh.red4[lane].x : 0.f);
+    if (lane < cs) st_cluster_f4(&sh.slot[parity][rank], uint32_t(lane), make_float4(cta, 0.f, 0.f, 0.f));
   }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, off));
-    md = fmaxf(md, __shfl_xor_sync(0xffffffffu, md, off));
+  cluster_sync();
+  return warp_sum_bcast(lane < cs ? sh.slot[parity][lane].x : 0.f);
+}
+
+// The rows' maxima and exponential sums over the cluster from each thread's
+// (m_t, s_t, m_d, s_d), s = sum 2^((x - m) k2): (Mt, Zt, Md, Zd). The same
+// three levels as a sum: warps, warp 0 over the warps, the CTAs.
+__device__ float4 spec_cluster_ms(SpecShared &sh, float4 v, int parity, int cs, uint32_t rank, float k2) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float4 w = ms4_lanes(v, k2);
+  if (lane == 0) sh.red4[warp] = w;
+  __syncthreads();
+  if (warp == 0) {
+    const float4 cta = ms4_lanes(lane < 16 ? sh.red4[lane] : make_float4(-INFINITY, 0.f, -INFINITY, 0.f), k2);
+    if (lane < cs) st_cluster_f4(&sh.slot[parity][rank], uint32_t(lane), cta);
   }
-  float zt = 0.f, zd = 0.f;
-  for (int i = lane; i < cs * 16; i += 32) {
-    const float4 e = sh.slot[parity][i];
-    if (e.x != -INFINITY) zt += e.y * exp2f_approx((e.x - mt) * k2);
-    if (e.z != -INFINITY) zd += e.w * exp2f_approx((e.z - md) * k2);
-  }
-  return make_float4(mt, warp_sum_bcast(zt), md, warp_sum_bcast(zd));
+  cluster_sync();
+  return ms4_lanes(lane < cs ? sh.slot[parity][lane] : make_float4(-INFINITY, 0.f, -INFINITY, 0.f), k2);
 }
 
 // Warp 0: the parent and token rows of a sequence into sh (entries past
 // tree_len: parent -1, token 0); DREAMS_DATA_BAD_PARENT when parent[0] != -1
-// or a parent[i] lies outside [0, i).
-__device__ int spec_tree_warp(SpecShared &sh, const int32_t *par_row, const int32_t *tok_row, int T) {
+// or a parent[i] lies outside [0, i). pre_par / pre_tok: the rows' first Tm
+// entries, loaded before tree_len was known.
+__device__ int spec_tree_warp(SpecShared &sh, const int (&pre_par)[2], const int (&pre_tok)[2], int T) {
   const int lane = threadIdx.x & 31;
   int bad = 0;
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int i = lane + 32 * h;
     const bool live = i < T;
-    const int pa = live ? __ldg(par_row + i) : -1;
+    const int pa = live ? pre_par[h] : -1;
     sh.par[i] = pa;
-    sh.tok[i] = live ? __ldg(tok_row + i) : 0;
+    sh.tok[i] = live ? pre_tok[h] : 0;
     if (i == 0) bad |= pa != -1;
     else if (live) bad |= pa < 0 || pa >= i;
   }
@@ -1327,20 +1350,35 @@ __device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed,
   }
   if (lane == 0) sh.last[warp] = last;
   __syncthreads();
-  int slast = -1;
-  for (int w = 0; w < 16; ++w) slast = max(slast, sh.last[w]);
+  // lane w < 16 holds warp w's values: maxima and sums across the lanes (the
+  // same bits in every warp)
+  int slast = lane < 16 ? sh.last[lane] : -1;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) slast = max(slast, __shfl_xor_sync(0xffffffffu, slast, off));
   if (tail || slast < 0) return slast;
-  // the crossing chunk (every thread walks the same sums in the same order)
+  // the crossing chunk: chunk totals, then their running sum in chunk order
   int jc = -1;
-  float before = 0.f;
-  for (int j = 0; j < J && jc < 0; ++j) {
-    float t = 0.f;
-    for (int w = 0; w < 16; ++w) t += sh.chunk[j][w];
-    if (t > 0.f && before + t > rem) jc = j;
-    else before += t;
+  float before = 0.f, cw = 0.f;  // cw: lane w's sum of chunk jc
+#pragma unroll
+  for (int j = 0; j < SPEC_MAX_J; ++j) {
+    if (j >= J) break;
+    const float v = lane < 16 ? sh.chunk[j][lane] : 0.f;
+    const float t = warp_sum_bcast(v);
+    if (jc < 0) {
+      if (t > 0.f && before + t > rem) jc = j, cw = v;
+      else before += t;
+    }
   }
   if (jc < 0) return slast;  // rounding: no crossing inside the slice
   rem -= before;
+  // this warp's offset in chunk jc: the sums of the warps before it
+  float wi = cw;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, wi, off);
+    if (lane >= off) wi += y;
+  }
+  const float wbase = __shfl_sync(0xffffffffu, wi - cw, warp);
   // exclusive scan of the threads' sums of chunk jc, in thread order
   float mine = 0.f;
 #pragma unroll
@@ -1352,15 +1390,14 @@ __device__ int spec_slice_draw(SpecShared &sh, const float *et, const float *ed,
     const float y = __shfl_up_sync(0xffffffffu, inc, off);
     if (lane >= off) inc += y;
   }
-  float wbase = 0.f;
-  for (int w = 0; w < warp; ++w) wbase += sh.chunk[jc][w];
   const float excl = wbase + inc - mine;
   const bool cross = mine > 0.f && excl + mine > rem;
   const unsigned bal = __ballot_sync(0xffffffffu, cross);
   if (lane == 0) sh.hit[warp] = bal ? warp * 32 + __ffs(bal) - 1 : INT_MAX;
   __syncthreads();
-  int th = INT_MAX;
-  for (int w = 0; w < 16; ++w) th = min(th, sh.hit[w]);
+  int th = lane < 16 ? sh.hit[lane] : INT_MAX;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) th = min(th, __shfl_xor_sync(0xffffffffu, th, off));
   if (th == INT_MAX) return slast;
   if (tid == th) {
     const int e0 = jc * SPEC_CHUNK + 8 * tid;
@@ -1404,12 +1441,24 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       asm volatile("prefetch.L2 [%0];" ::"l"(dp));
     }
   }
+  // the tree rows go out with the lengths (rows of T_max entries exist)
+  int pre_par[2] = {-1, -1}, pre_tok[2] = {0, 0};
+  if (warp == 0) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int i = lane + 32 * h;
+      if (i < Tm) {
+        pre_par[h] = ld_issue_now(p.tr.parent + rb + i);
+        pre_tok[h] = ld_issue_now(p.tr.tokens + rb + i);
+      }
+    }
+  }
   const int TL = __ldg(p.tr.tree_len + b), L = __ldg(p.tr.kv_len + b);
   if (warp == 0) {
     int bad = 0;
     if (TL < 1 || TL > Tm) bad = DREAMS_DATA_BAD_TREE_LEN;
     else if (L < 0 || L > p.kv.capacity - TL) bad = DREAMS_DATA_BAD_KV_LEN;
-    else bad = spec_tree_warp(sh, p.tr.parent + rb, p.tr.tokens + rb, TL);
+    else bad = spec_tree_warp(sh, pre_par, pre_tok, TL);
     if (lane == 0) {
       sh.cmd = bad;
       if (bad && rank == 0) flag(p.status, bad);
@@ -1432,16 +1481,24 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       const bool try_kids = kids != 0 && n < p.max_path - 1;
       // each child's logits at its draft token and its uniform, loaded while
       // the rows are (children have larger indices than every node read before)
-      if (try_kids && tid < 64 && ((kids >> tid) & 1)) {
+      const bool my_kid = try_kids && tid < 64 && ((kids >> tid) & 1);
+      float kid_t = -INFINITY, kid_d = -INFINITY, kid_u = 0.f;
+      if (my_kid) {
         const int x = sh.tok[tid];
-        const bool in = x >= 0 && x < p.V;
-        sh.cxt[tid] = in ? __uint_as_float(Elem<T>::bits(trow, x)) : -INFINITY;
-        sh.cxd[tid] = in ? __uint_as_float(Elem<T>::bits(drow, x)) : -INFINITY;
-        sh.cu[tid] = __ldg(p.u_acc + rb + tid);
+        if (x >= 0 && x < p.V) {
+          kid_t = ld_now_val<T>(trow + x);
+          kid_d = ld_now_val<T>(drow + x);
+        }
+        kid_u = ld_now_f32(p.u_acc + rb + tid);
       }
-      const float u_bonus = __ldg(p.u_res + rb + cur);
+      const float u_bonus = ld_now_f32(p.u_res + rb + cur);
       // the rows' maxima and exponential sums: per thread, then over the cluster
       const float2 m = spec_load_rows<T>(p, trow, drow, try_kids, v0, et, ed);
+      if (my_kid) {  // stored after the rows' loads are out
+        sh.cxt[tid] = kid_t;
+        sh.cxd[tid] = kid_d;
+        sh.cu[tid] = kid_u;
+      }
       const float st = spec_exp_inplace(et, m.x, k2, J);
       const float sd = try_kids ? spec_exp_inplace(ed, m.y, k2, J) : 0.f;
       const float4 g = spec_cluster_ms(sh, make_float4(m.x, st, m.y, sd), parity, cs, rank, k2);
@@ -1495,27 +1552,36 @@ __global__ void __launch_bounds__(SPEC_THREADS) spec_walk_kernel(const SpecParam
       float wj[SPEC_MAX_J];
       int last;
       const float tot = spec_weights(et, ed, at, ct, use_q, J, wj, last);
-      spec_push(sh, make_float4(warp_sum_bcast(tot), 0.f, 0.f, 0.f), parity, cs, rank);
-      // per-slice totals (lane r: slice r, its warps in order), then the
-      // crossing slice, the same on every warp of every CTA
-      float tr = 0.f;
-      if (lane < cs)
-        for (int w = 0; w < 16; ++w) tr += sh.slot[parity][lane * 16 + w].x;
+      // the slice's total (warps, then warp 0 over them) to slot [parity][rank]
+      // of every CTA; lane r then holds slice r's total, the same bits on
+      // every warp of every CTA
+      {
+        const float wt = warp_sum_bcast(tot);
+        if (lane == 0) sh.red[warp] = wt;
+        __syncthreads();
+        if (warp == 0) {
+          const float slice = warp_sum_bcast(lane < 16 ? sh.red[lane] : 0.f);
+          if (lane < cs) st_cluster_f4(&sh.slot[parity][rank], uint32_t(lane), make_float4(slice, 0.f, 0.f, 0.f));
+        }
+        cluster_sync();
+      }
+      const float tr = lane < cs ? sh.slot[parity][lane].x : 0.f;
       parity ^= 1;
-      float total = 0.f;
-      for (int r = 0; r < cs; ++r) total += __shfl_sync(0xffffffffu, tr, r);
+      // their running sum across the lanes, then the crossing slice
+      float inc = tr;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, inc, off);
+        if (lane >= off) inc += y;
+      }
+      const float total = __shfl_sync(0xffffffffu, inc, 31);
       const float u = u_bonus > 0.f ? fminf(u_bonus, 1.f) : 0.f;
       const float target = u * total;
-      int cr = -1, lastpos = -1;
-      float before = 0.f;
-      for (int r = 0; r < cs; ++r) {
-        const float t = __shfl_sync(0xffffffffu, tr, r);
-        if (t > 0.f) lastpos = r;
-        if (cr < 0) {
-          if (t > 0.f && before + t > target) cr = r;
-          else before += t;
-        }
-      }
+      const unsigned pos = __ballot_sync(0xffffffffu, tr > 0.f);
+      const unsigned crs = __ballot_sync(0xffffffffu, tr > 0.f && inc > target);
+      int cr = crs ? __ffs(crs) - 1 : -1;
+      const int lastpos = pos ? 31 - __clz(pos) : -1;
+      const float before = __shfl_sync(0xffffffffu, inc - tr, cr >= 0 ? cr : 0);
       const bool tail = cr < 0;
       if (tail) cr = lastpos;
       if (cr < 0) {  // no positive weight anywhere (rounding): token 0
