@@ -136,6 +136,7 @@ struct TcParams {
   CUtensorMap tmap_q;
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;
+  CUtensorMap tmap_o;  // the output, with the query block's box
   AttnParams a;
   int32_t paged;
 };
@@ -252,7 +253,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   __shared__ __align__(8) uint64_t bar_kf[NK], bar_ke[NK], bar_vf[NV], bar_ve[NV];
   __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_q, bar_drain, bar_never;
   __shared__ uint32_t s_tmem;
-  __shared__ int s_abort, s_zero, s_flag;
+  __shared__ int s_abort, s_zero, s_flag, s_tma;
   __shared__ unsigned long long s_anc[64];
   __shared__ int s_jump[64];
   __shared__ int s_key[RANK_PAIRS];
@@ -830,9 +831,16 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       s_ml[wg * ROWS + row] = make_float2(m_ref, l);
       if (ENT) s_w[wg * ROWS + row] = wsum;
     }
+    // A block whose every row inside the tensor is a real query row leaves
+    // through one TMA store per 64-column region (the box of the Q map, over
+    // the output): the rows are staged in shared memory in the box's 128-byte
+    // swizzled layout (the first K stage, idle once every MMA has completed).
+    // Other blocks store row by row (rows past tree_len / q_len stay untouched).
+    if (tid == 0) s_tma = direct && ::min(t0 + p.TB, p.T_max) <= T && !*abort_flag;
     tc::fence_before_sync();
     named_sync(1, 256);
     tc::fence_after_sync();
+    const bool tma_out = s_tma != 0;
     const int64_t slot = (((int64_t(b) * p.Hkv + g) * p.nrb + rb) * p.nsplit + split) * ROWS;
     if (act && !*abort_flag) {
       const float2 a = s_ml[row], c = s_ml[ROWS + row];
@@ -856,6 +864,19 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           const float va = ca != 0.f ? ca * __uint_as_float(oa[e]) : 0.f;
           const float vb = cb != 0.f ? cb * __uint_as_float(ob[e]) : 0.f;
           o[e] = (va + vb) * inv;
+        }
+        if (tma_out) {
+          // region col / 64, 16-byte chunk (col % 64) / 8 + e of row `row`
+          const uint32_t rbase = k_s(0) + uint32_t((col >> 6) * Q_REGION + row * 128);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int c = ((col & 63) >> 3) + e;
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(rbase + uint32_t((c ^ (row & 7)) << 4)),
+                         "r"(pack_bf16x2(o[8 * e], o[8 * e + 1])), "r"(pack_bf16x2(o[8 * e + 2], o[8 * e + 3])),
+                         "r"(pack_bf16x2(o[8 * e + 4], o[8 * e + 5])), "r"(pack_bf16x2(o[8 * e + 6], o[8 * e + 7]))
+                         : "memory");
+          }
+          continue;
         }
         if (!real_row) continue;
         if (direct) {
@@ -890,6 +911,16 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     } else if (act && *abort_flag == 1 && !direct && wg == 0 && real_row) {
       // a wait gave up: the negative sum tells the merge to leave the row alone
       p.ws_ml[slot + row] = make_float2(-INFINITY, -1.f);
+    }
+    if (tma_out) {
+      tc::fence_proxy_async_smem();  // the staged rows, to the TMA engine
+      named_sync(1, 256);
+      if (tid == 0) {
+#pragma unroll
+        for (int r = 0; r < NR; ++r) tc::tma_store_5d(&P.tmap_o, k_s(0) + r * Q_REGION, r * 64, 0, g, t0, b);
+        tc::bulk_commit_group();
+        tc::bulk_wait_group_read0();  // shared memory stays until the copy engine has read it
+      }
     }
   }
 
@@ -1145,7 +1176,9 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   P.a = a;
   P.paged = kv->page_table != nullptr;
   if (!make_kv_map(&P.tmap_k, k, kv, B) || !make_kv_map(&P.tmap_v, v, kv, B) ||
-      !make_q_map(&P.tmap_q, a.q, B, a.T_max, a.Hq, a.Hkv, D, a.TB, q_stride_b, q_stride_t))
+      !make_q_map(&P.tmap_q, a.q, B, a.T_max, a.Hq, a.Hkv, D, a.TB, q_stride_b, q_stride_t) ||
+      !make_q_map(&P.tmap_o, a.out, B, a.T_max, a.Hq, a.Hkv, D, a.TB, int64_t(a.T_max) * a.Hq * D,
+                  int64_t(a.Hq) * D))
     return DREAMS_ERR_UNSUPPORTED;
   if (pl.ordered) {
     tree_attn_order_kernel<<<1, ORDER_THREADS, 0, stream>>>(a);
