@@ -305,3 +305,53 @@ def test_speculative_repeatable(dreams):
     torch.cuda.synchronize()
     for key in a:
         assert torch.equal(a[key], b[key]), key
+
+
+def test_speculative_multi_layer_paged_cache(dreams):
+    """Three layer caches in 64-slot pages (a permuted page table), random bit
+    patterns in every slot (NaN bf16 included): each cluster moves the accepted
+    nodes' K/V of every layer and head; all other bytes are unchanged. One
+    sequence's page table points outside the pool: it is flagged, its cache is
+    left alone, and the walk outputs are still written."""
+    rng = np.random.default_rng(66)
+    B, T, V, Hkv, D, n_layers, page, pps = 6, 20, 1500, 2, 64, 3, 64, 3
+    cap = pps * page
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    tl = np.full(B, T, np.int32)
+    tgt = (2.0 * rng.standard_normal((B, T, V))).astype(np.float32)
+    drf = (tgt + 0.5 * rng.standard_normal((B, T, V))).astype(np.float32)
+    tok = _draft_tokens(rng, drf, par, tl, 1.0)
+    kl = rng.integers(0, cap - T + 1, B).astype(np.int32)
+    table = rng.permutation(B * pps).astype(np.int32).reshape(B, pps)
+    kin = rng.integers(0, 65536, (n_layers, B * pps, page, Hkv, D), dtype=np.uint16)
+    vin = rng.integers(0, 65536, (n_layers, B * pps, page, Hkv, D), dtype=np.uint16)
+    u_acc, u_res, ref = _oracle_clean(tgt, drf, par, tok, tl, kl, 6, 1.0, rng)
+    lay = oracle.KVLayout(cap, Hkv, D, page_table=table, page_size=page, num_pages=B * pps)
+    ko, vo, ost = oracle.kv_compact(kin, vin, lay, kl, ref["accept_len"], ref["path"], n_layers=n_layers,
+                                    layer_stride=kin[0].size)
+    assert ost == 0
+    tk = torch.from_numpy(kin.view(np.int16)).view(torch.bfloat16).cuda()
+    tv = torch.from_numpy(vin.view(np.int16)).view(torch.bfloat16).cuda()
+    r, st = _run(dreams, torch.from_numpy(tgt).cuda(), torch.from_numpy(drf).cuda(), par, tok, tl, kl, tk, tv, 6,
+                 1.0, u_acc, u_res, torch.from_numpy(table).cuda())
+    assert st == 0
+    _compare(r, ref)
+    assert np.array_equal(tk.view(torch.int16).cpu().numpy().view(np.uint16), ko)
+    assert np.array_equal(tv.view(torch.int16).cpu().numpy().view(np.uint16), vo)
+    # a page id outside the pool in a sequence whose walk moves rows
+    moved = int(np.argmax(ref["accept_len"]))
+    assert ref["accept_len"][moved] >= 2
+    bad = table.copy()
+    bad[moved, :] = B * pps + 5
+    tk2 = torch.from_numpy(kin.view(np.int16)).view(torch.bfloat16).cuda()
+    tv2 = torch.from_numpy(vin.view(np.int16)).view(torch.bfloat16).cuda()
+    r2, st2 = _run(dreams, torch.from_numpy(tgt).cuda(), torch.from_numpy(drf).cuda(), par, tok, tl, kl, tk2, tv2, 6,
+                   1.0, u_acc, u_res, torch.from_numpy(bad).cuda())
+    assert st2 & dreams.DATA_BAD_PAGE
+    _compare(r2, ref)
+    acc_ok = ref["accept_len"].copy()
+    acc_ok[moved] = 1  # nothing moves for the flagged sequence
+    ko2, vo2, _ = oracle.kv_compact(kin, vin, lay, kl, acc_ok, ref["path"], n_layers=n_layers,
+                                    layer_stride=kin[0].size)
+    assert np.array_equal(tk2.view(torch.int16).cpu().numpy().view(np.uint16), ko2)
+    assert np.array_equal(tv2.view(torch.int16).cpu().numpy().view(np.uint16), vo2)
