@@ -387,12 +387,15 @@ def run_dreams(args, rank, world, local):
         try:
             captured = []
             for c in copies:
-                ga, gs = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+                ga, gs, gf = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
                 with torch.cuda.graph(ga):
                     attn_call(c)
                 with torch.cuda.graph(gs):
                     step_call(c)
-                captured.append((ga, gs))
+                with torch.cuda.graph(gf):  # the whole step, as a serving loop would replay it
+                    attn_call(c)
+                    step_call(c)
+                captured.append((ga, gs, gf))
             graphs = captured
             stream = torch.cuda.current_stream(dev)
             for i in range(2):
@@ -400,7 +403,7 @@ def run_dreams(args, rank, world, local):
             torch.cuda.synchronize(dev)
             if int(status.item()) != 0:
                 raise RuntimeError(f"device status {int(status.item()):#x} on valid input (graph replay)")
-            launch_mode = "cuda-graph replay"
+            launch_mode = "cuda-graph replay (one graph per step)"
         except RuntimeError as e:  # capture unsupported here: time eager launches instead
             if "device status" in str(e):
                 raise
@@ -416,29 +419,55 @@ def run_dreams(args, rank, world, local):
         torch.cuda.synchronize(dev)
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
     flush_buf = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev) if args.flush_l2 else None
     flush_read = torch.zeros(L2_BYTES // 2, dtype=torch.float32, device=dev) if args.flush_l2 else None
+
+    def flush():
+        # the write evicts the step's inputs; the read then evicts the dirty
+        # lines, so the step pays no write-back of the flush
+        flush_buf.fill_(0xA5)
+        flush_read.sum()
+
+    # the timed steps: each input copy's whole step (attention, then the
+    # verification tail) as one graph; back to back, the timed span over K;
+    # with flushes between steps, the mean of the steps' own spans
+    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     barrier()
     t0 = time.time()
     for i in range(K):
         if flush_buf is not None:
-            # the write evicts the step's inputs; the read then evicts the
-            # dirty lines, so the step pays no write-back of the flush
-            flush_buf.fill_(i & 255)
-            flush_read.sum()
-        step(i % 2, evs[i])
+            flush()
+        if flush_buf is not None or i == 0:
+            sev[i][0].record(stream)
+        if graphs is not None:
+            graphs[i % 2][2].replay()
+        else:
+            attn_call(copies[i % 2])
+            step_call(copies[i % 2])
+        if flush_buf is not None or i == K - 1:
+            sev[i][1].record(stream)
     barrier()
     wall = time.time() - t0
     clk = clocks.stop()
+    if flush_buf is None:
+        ms_per_step = sev[0][0].elapsed_time(sev[-1][1]) / K
+    else:
+        ms_per_step = sum(e[0].elapsed_time(e[1]) for e in sev) / K
+    ms_per_step = max_over_ranks(ms_per_step, dev)
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item()):#x} on valid input (timed steps)")
 
-    total_ms = evs[0][0].elapsed_time(evs[-1][2])
+    # the split between the attention and the tail: the same steps with an
+    # event between the two calls (separate graphs), timed after the headline
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    barrier()
+    for i in range(K):
+        if flush_buf is not None:
+            flush()
+        step(i % 2, evs[i])
+    barrier()
     attn_ms = [e[0].elapsed_time(e[1]) for e in evs]
     tail_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    # back to back: the whole timed span over K; with the flushes between
-    # steps: the mean of the steps' own spans
-    ms_per_step = total_ms / K if flush_buf is None else sum(e[0].elapsed_time(e[2]) for e in evs) / K
-    ms_per_step = max_over_ranks(ms_per_step, dev)
 
     # ---- e2e through the public API with host buffers. The inputs of a step
     # are the tree arrays and the q and logits rows of its real tree nodes
