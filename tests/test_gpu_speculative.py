@@ -355,3 +355,33 @@ def test_speculative_multi_layer_paged_cache(dreams):
                                     layer_stride=kin[0].size)
     assert np.array_equal(tk2.view(torch.int16).cpu().numpy().view(np.uint16), ko2)
     assert np.array_equal(tv2.view(torch.int16).cpu().numpy().view(np.uint16), vo2)
+
+
+@pytest.mark.parametrize("B, V, sigma", [(2, 128256, 2.0), (3, 256000, 4.0)])
+def test_speculative_clusters_of_16(dreams, B, V, sigma):
+    """Clusters of 16 CTAs: a batch of at most 4 over a 128256-entry
+    vocabulary (16 CTAs per sequence to spread the passes), and a 256000-entry
+    vocabulary, whose rows need 16 slices of shared memory (the non-portable
+    cluster size). A draw's margin is at most half the width of the entry it
+    lands in, so the larger vocabulary takes more peaked rows (sigma 4), whose
+    draws land in entries of percent-level width."""
+    rng = np.random.default_rng(B * 7 + V % 97)
+    T, cap = 24, 64
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    tl = np.full(B, T, np.int32)
+    tgt32 = (sigma * rng.standard_normal((B, T, V))).astype(np.float32)
+    drf32 = (tgt32 + 0.5 * rng.standard_normal((B, T, V))).astype(np.float32)
+    tgt_t, drf_t = W.bf16(tgt32), W.bf16(drf32)
+    del tgt32, drf32
+    tok = _draft_tokens(rng, drf_t.float().numpy(), par, tl, 1.0)
+    kl = rng.integers(0, cap - T + 1, B).astype(np.int32)
+    u_acc, u_res, ref = _oracle_clean(W.bits(tgt_t), W.bits(drf_t), par, tok, tl, kl, 6, 1.0, rng, bf16=True)
+    k = W.bf16(rng.standard_normal((B, cap, 1, 64), dtype=np.float32))
+    kg, vg = k.cuda(), k.clone().cuda()
+    r, st = _run(dreams, tgt_t.cuda(), drf_t.cuda(), par, tok, tl, kl, kg, vg, 6, 1.0, u_acc, u_res)
+    assert st == 0
+    _compare(r, ref)
+    assert (ref["accept_len"] >= 2).any()
+    ko, _, ost = oracle.kv_compact(W.bits(k), W.bits(k), oracle.KVLayout(cap, 1, 64), kl, ref["accept_len"],
+                                   ref["path"])
+    assert ost == 0 and np.array_equal(W.bits(kg.cpu()), ko)
