@@ -218,3 +218,29 @@ def test_binding_checks_before_any_call():
         dreams._q_strides(q)
     fused = torch.zeros((2, 5, 3, 4, 64), dtype=torch.bfloat16)
     assert dreams._q_strides(fused[:, :, 0]) == (5 * 3 * 4 * 64, 3 * 4 * 64)
+
+
+def test_speculative_binding_checks_before_any_call():
+    """verify_step_speculative refuses on the host, before any library call:
+    target and draft logits of different dtypes or shapes, rows that are not
+    [B, T_max, V] with contiguous rows, logits of another dtype, and uniforms
+    of the wrong shape or dtype."""
+    B, T, V = 2, 4, 16
+    tree = dreams.Tree(torch.full((B, T), -1, dtype=torch.int32), torch.zeros((B, T), dtype=torch.int32),
+                       torch.ones(B, dtype=torch.int32), torch.zeros(B, dtype=torch.int32))
+    k = torch.zeros((B, 8, 1, 64), dtype=torch.bfloat16)
+    kv = dreams.KVCache(k, k.clone())
+    tgt = torch.zeros((B, T, V), dtype=torch.float32)
+    u = torch.zeros((B, T), dtype=torch.float32)
+    with pytest.raises(ValueError, match="share dtype, shape and strides"):
+        dreams.verify_step_speculative(tgt, tgt.to(torch.bfloat16).float()[:, :, :8], tree, kv, 3, 1.0, u, u)
+    with pytest.raises(ValueError, match="share dtype, shape and strides"):
+        dreams.verify_step_speculative(tgt, tgt.to(torch.bfloat16), tree, kv, 3, 1.0, u, u)
+    with pytest.raises(ValueError, match="uniformly strided contiguous rows"):
+        dreams.verify_step_speculative(tgt.transpose(1, 2), tgt.transpose(1, 2), tree, kv, 3, 1.0, u, u)
+    with pytest.raises(TypeError, match="float32/bfloat16"):
+        dreams.verify_step_speculative(tgt.double(), tgt.double(), tree, kv, 3, 1.0, u, u)
+    with pytest.raises(ValueError, match=r"u_accept must be \[B, T_max\]"):
+        dreams.verify_step_speculative(tgt, tgt, tree, kv, 3, 1.0, torch.zeros((B, 2), dtype=torch.float32), u)
+    with pytest.raises((TypeError, ValueError)):
+        dreams.verify_step_speculative(tgt, tgt, tree, kv, 3, 1.0, u, u.double())
