@@ -240,7 +240,8 @@ def time_workload(dreams, dev, name: str, K: int, status, barrier) -> dict:
     """Step, attention and verification-tail times of one workload, the same
     calls as the headline step: two input copies, each copy's whole step
     captured as one CUDA graph (the step time) and its two calls as two (the
-    split), CUDA events on the launching stream. These workloads fit in L2, so
+    split), CUDA events on the launching stream; then the speculative-sampling
+    tail at temperature 1. These workloads fit in L2, so
     before every step (outside its events) a buffer twice the size of L2 is
     written, then another as large as L2 read; the per-step times are
     averaged."""
@@ -313,10 +314,45 @@ def time_workload(dreams, dev, name: str, K: int, status, barrier) -> dict:
         fev[i][1].record(stream)
     barrier()
     s_us = sum(e[0].elapsed_time(e[1]) for e in fev) / K * 1000.0
+    # the speculative-sampling tail (temperature 1, draft = target + N(0, 0.5)
+    # noise), one graph per input copy, the same flush before every step
+    g = torch.Generator(device=dev).manual_seed(11)
+    drafts = [(c["logits"].float() + 0.5 * torch.randn(c["logits"].shape, generator=g, device=dev)).to(
+        c["logits"].dtype) for c in copies]
+    cpu_g = torch.Generator().manual_seed(13)
+    u_a = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
+    u_r = torch.rand((w.B, w.T_max), generator=cpu_g).to(dev)
+
+    def spec_call(i):
+        c = copies[i]
+        dreams.verify_step_speculative(c["logits"], drafts[i], c["tree"], c["kv"], w.max_path, 1.0, u_a, u_r,
+                                       outputs=c["outs"], status=status)
+
+    for i in range(4):
+        spec_call(i % 2)
+    sgraphs = []
+    for i in range(2):
+        gsp = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gsp):
+            spec_call(i)
+        sgraphs.append(gsp)
+    pev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+    barrier()
+    for i in range(K):
+        flush_buf.fill_(i & 255)
+        flush_read.sum()
+        pev[i][0].record(stream)
+        sgraphs[i % 2].replay()
+        pev[i][1].record(stream)
+    barrier()
+    sp_us = sum(e[0].elapsed_time(e[1]) for e in pev) / K * 1000.0
+    sp_acc = sum(float(c["outs"][0].float().mean()) for c in copies) / 2  # both copies were replayed
+    del drafts, sgraphs
     ab, gb = attn_bytes(w), argmax_bytes(w)
     return {"workload": w.spec.description, "attn_us": round(a_us, 2), "attn_bytes": ab,
             "attn_GBps": round(ab / (a_us * 1e-6) / 1e9, 1), "verify_us": round(v_us, 2), "argmax_bytes": gb,
             "verify_argmax_GBps": round(gb / (v_us * 1e-6) / 1e9, 1), "step_us": round(s_us, 2),
+            "speculative_us": round(sp_us, 2), "speculative_mean_accept_len": round(sp_acc, 3),
             "launch": "cuda-graph replay", "l2": "flushed before every step (outside its events)", "steps": K}
 
 

@@ -385,3 +385,23 @@ def test_speculative_clusters_of_16(dreams, B, V, sigma):
     ko, _, ost = oracle.kv_compact(W.bits(k), W.bits(k), oracle.KVLayout(cap, 1, 64), kl, ref["accept_len"],
                                    ref["path"])
     assert ost == 0 and np.array_equal(W.bits(kg.cpu()), ko)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_speculative_llava_f32_temperature_1(dreams, seed):
+    """The LLaVA-7B-shaped workload (f32 logits over 32000 entries, one
+    sequence, a cluster of 8 CTAs) at temperature 1, drafts = target + N(0, 0.5)
+    noise, against the oracle."""
+    w = W.make("llava7b", with_attn=False)
+    rng = np.random.default_rng(500 + seed)
+    tgt = w.logits.numpy()
+    drf = (tgt + 0.5 * rng.standard_normal(tgt.shape, dtype=np.float32)).astype(np.float32)
+    par, tok, tl, kl = (x.numpy() for x in (w.parent, w.tokens, w.tree_len, w.kv_len))
+    u_acc, u_res, ref = _oracle_clean(tgt, drf, par, tok, tl, kl, w.max_path, 1.0, rng)
+    assert ref["status"] == 0
+    cap = int(kl.max()) + w.T_max
+    k = torch.zeros((w.B, cap, 1, 8), dtype=torch.bfloat16, device="cuda")
+    r, st = _run(dreams, torch.from_numpy(tgt).cuda(), torch.from_numpy(drf).cuda(), par, tok, tl, kl, k, k.clone(),
+                 w.max_path, 1.0, u_acc, u_res)
+    assert st == 0
+    _compare(r, ref)
