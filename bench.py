@@ -654,6 +654,46 @@ def run_dreams(args, rank, world, local):
                    "launch": sampled_mode, "GBps": round(argmax_bytes(w) / (sampled_us * 1e-6) / 1e9, 1)}
         del sampled_graphs
 
+    # ---- the argmax kernel alone (dreams_vocab_argmax) over every row of the
+    # logits [B * T_max, V], padding rows included (all of them are read), the
+    # two input copies alternating (each larger than L2), graph replay
+    rows_all = w.B * w.T_max
+    am_out = torch.empty(rows_all, dtype=torch.int32, device=dev)
+    am_ws = torch.zeros(max(16, int(dreams._lib().dreams_vocab_argmax_workspace_size(rows_all, w.V))),
+                        dtype=torch.uint8, device=dev)
+
+    def am_call(i):
+        dreams.vocab_argmax(copies[i % 2]["logits"], out=am_out, workspace=am_ws)
+
+    for i in range(4):
+        am_call(i)
+    am_graphs = None
+    if not args.no_graph:
+        am_graphs = []
+        for i in range(2):
+            gam = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gam):
+                am_call(i)
+            am_graphs.append(gam)
+    Ka = max(3, min(K, 100))
+    s0 = torch.cuda.Event(enable_timing=True)
+    s1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    s0.record(stream)
+    for i in range(Ka):
+        if am_graphs is not None:
+            am_graphs[i % 2].replay()
+        else:
+            am_call(i)
+    s1.record(stream)
+    barrier()
+    am_us = s0.elapsed_time(s1) / Ka * 1000.0
+    am_bytes = rows_all * w.V * w.logits.element_size()
+    argmax_alone = {"us": round(am_us, 2), "bytes": am_bytes, "GBps": round(am_bytes / (am_us * 1e-6) / 1e9, 1),
+                    "rows": rows_all, "launch": "cuda-graph replay" if am_graphs is not None else "eager",
+                    "note": "every row of [B*T_max, V], padding rows included; the two copies alternate"}
+    del am_graphs
+
     # ---- speculative sampling over the tree at temperature 1: draft logits =
     # target + N(0, 0.5) noise, drafts accepted with probability min(1, r/q)
     speculative = None
@@ -867,6 +907,9 @@ def run_dreams(args, rank, world, local):
         "verify_step": {"us": round(tail_avg_ms * 1000, 2), "argmax_bytes": gb, "GBps": round(tail_gbs, 1),
                         "frac_measured_hbm": round(tail_gbs / peak, 4)},
     }
+    argmax_alone["frac_measured_hbm"] = round(argmax_alone["GBps"] / peak, 4)
+    argmax_alone["frac_of_nominal_8000"] = round(argmax_alone["GBps"] / NOMINAL_HBM_GBS, 4)
+    kernels["vocab_argmax"] = argmax_alone
     if sampled is not None:
         sampled["frac_measured_hbm"] = round(sampled["GBps"] / peak, 4)
         kernels["verify_step_sampled"] = sampled
