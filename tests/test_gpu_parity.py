@@ -446,6 +446,39 @@ def test_verify_step_matches_oracle(dreams, name):
     assert np.array_equal(W.bits(g["v"].cpu()), vo)
 
 
+@pytest.mark.parametrize("name", ["batched", "llava7b"])
+def test_verify_step_per_sequence_views(dreams, name):
+    """verify_step called once per sequence, on views of that sequence's row
+    of every input and output (a KV cache view: its page-table row, or its
+    slice of a contiguous cache), gives what one batched call gives: the same
+    predictions, walk outputs and compacted cache, bit for bit. The bench's
+    end-to-end step verifies each sequence as its logits land this way."""
+    w = W.make(name)
+    a, b_ = to_gpu(w), to_gpu(w)
+    st = _status()
+    am_a = torch.full((w.B, w.T_max), -7, dtype=torch.int32, device="cuda")
+    r_a = dreams.verify_step(a["logits"], a["tree"], a["kv"], w.max_path, argmax_out=am_a, status=st)
+    am_b = torch.full((w.B, w.T_max), -7, dtype=torch.int32, device="cuda")
+    outs = (torch.full((w.B,), -9, dtype=torch.int32, device="cuda"),
+            torch.full((w.B, w.max_path), -9, dtype=torch.int32, device="cuda"),
+            torch.full((w.B, w.max_path), -9, dtype=torch.int32, device="cuda"),
+            torch.full((w.B,), -9, dtype=torch.int32, device="cuda"))
+    tr = b_["tree"]
+    for s in range(w.B):
+        one = slice(s, s + 1)
+        kv_s = (dreams.KVCache(b_["k"], b_["v"], b_["page_table"][one]) if b_["page_table"] is not None
+                else dreams.KVCache(b_["k"][one], b_["v"][one]))
+        tree_s = dreams.Tree(tr.parent[one], tr.tokens[one], tr.tree_len[one], tr.kv_len[one])
+        dreams.verify_step(b_["logits"][one], tree_s, kv_s, w.max_path, argmax_out=am_b[one],
+                           outputs=tuple(o[one] for o in outs), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert torch.equal(am_a, am_b)
+    for key, o in zip(("accept_len", "path", "out_tokens", "new_kv_len"), outs):
+        assert torch.equal(r_a[key], o), key
+    assert torch.equal(a["k"], b_["k"]) and torch.equal(a["v"], b_["v"])
+
+
 def test_verify_step_bad_sequences(dreams):
     """Bad data in one sequence is reported and leaves the others intact."""
     w = W.make("batched", with_attn=True)
