@@ -538,7 +538,7 @@ def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path:
                         status: Optional[torch.Tensor] = None, stream=None) -> dict:
     """The verification tail at temperature > 0: the target's draw per tree
     node (``uniforms``: f32 [B, T_max]) takes the place of the argmax, then
-    acceptance and KV compaction, in one call (two kernel launches)."""
+    acceptance and KV compaction, in one call (three kernel launches)."""
     dev = tree.parent.device
     if logits.dtype not in (torch.float32, torch.bfloat16) or logits.device != dev:
         raise TypeError("logits must be float32/bfloat16 on the tree's device")
