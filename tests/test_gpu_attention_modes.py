@@ -85,3 +85,49 @@ def test_entropy_closed_forms(dreams):
     _, _, e_causal = _run(dreams, q, k[:, :T].contiguous(), v[:, :T].contiguous(), [T], [0], 0.125,
                           dreams.ATTN_CAUSAL)
     np.testing.assert_allclose(e_causal[0], np.log(np.arange(1, T + 1))[:, None].repeat(H, 1), atol=1e-4)
+
+
+def _paged(k, v, seed):
+    """The same cache as a pool of 64-slot pages in a seeded random order,
+    with its page table."""
+    B, cap, Hkv, D = k.shape
+    pps = cap // 64
+    perm = torch.randperm(B * pps, generator=torch.Generator().manual_seed(seed))
+    kp = torch.empty((B * pps, 64, Hkv, D), dtype=k.dtype)
+    vp = torch.empty_like(kp)
+    table = perm.view(B, pps).to(torch.int32)
+    for b in range(B):
+        for p in range(pps):
+            kp[table[b, p]] = k[b, 64 * p:64 * (p + 1)]
+            vp[table[b, p]] = v[b, 64 * p:64 * (p + 1)]
+    return kp, vp, table
+
+
+@pytest.mark.parametrize("mode", ["full", "causal"])
+def test_attention_modes_paged_equal_contiguous(dreams, mode):
+    """Cross-attention and causal prefill on a paged cache (pages in a random
+    order, several sequences of different lengths, a split KV range): the same
+    output, lse and entropy bits as on the contiguous cache, and the oracle's
+    values."""
+    B, Hq, Hkv, D, cap = 3, 8, 2, 128, 2048
+    causal = mode == "causal"
+    T_max = 300 if causal else 24
+    q, k, v = _case(77 if causal else 78, B, T_max, Hq, Hkv, D, cap)
+    q_len = [300, 129, 1] if causal else [24, 5, 1]
+    kv_len = [1500, 0, 1747] if causal else [2048, 700, 1]
+    m = dreams.ATTN_CAUSAL if causal else dreams.ATTN_FULL
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ql = torch.tensor(q_len, dtype=torch.int32, device="cuda")
+    kl = torch.tensor(kv_len, dtype=torch.int32, device="cuda")
+    kp, vp, table = _paged(k, v, 5)
+    res = []
+    for kvc in (dreams.KVCache(k.cuda(), v.cuda(), None), dreams.KVCache(kp.cuda(), vp.cuda(), table.cuda())):
+        res.append(dreams.attention(q.cuda(), kvc, ql, kl, D ** -0.5, m, want_lse=True, want_entropy=True, status=st))
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for b in range(B):
+        t = q_len[b]
+        for x, y in zip(res[0], res[1]):
+            assert torch.equal(x[b, :t], y[b, :t])
+    got = tuple(x.float().cpu().numpy() for x in res[1])
+    _compare(q, k, v, q_len, kv_len, D ** -0.5, causal, got, np.random.default_rng(3))
