@@ -696,10 +696,12 @@ __device__ TreeShape tree_shape_warp(const int32_t *par_row, const int32_t *tok_
 // The walk over a valid tree shape, one warp: a node matches when its draft
 // token equals its parent's prediction (the root always matches); a node is
 // accepted when every node of its root path matches. Writes the accepted
-// path into s_path[0..n]. Pred rows may have been written by other CTAs of
-// this grid or by the preceding grid, so they are read through L2.
+// path into s_path[0..n] and, when s_out is given, the tokens the step emits
+// into s_out[0..n] (the accepted drafts' tokens, from the shape's registers,
+// then the bonus prediction). Pred rows may have been written by other CTAs
+// of this grid or by the preceding grid, so they are read through L2.
 __device__ WalkOut tree_walk_finish(const TreeShape &ts, const int32_t *pred_row, int T, int max_path,
-                                    int32_t *s_path) {
+                                    int32_t *s_path, int32_t *s_out = nullptr) {
   __shared__ int s_pred[64];
   const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -741,8 +743,14 @@ __device__ WalkOut tree_walk_finish(const TreeShape &ts, const int32_t *pred_row
     const unsigned lo = __ballot_sync(0xffffffffu, ts.par[0] == cur && ((mark >> lane) & 1ull));
     const unsigned hi = __ballot_sync(0xffffffffu, ts.par[1] == cur && ((mark >> (lane + 32)) & 1ull));
     cur = lo ? (__ffs(lo) - 1) : (__ffs(hi) + 31);
-    if (lane == 0) s_path[k] = cur;
+    // node cur's token sits in lane cur % 32, slot cur / 32
+    const int tk = __shfl_sync(0xffffffffu, cur < 32 ? ts.tok[0] : ts.tok[1], cur & 31);
+    if (lane == 0) {
+      s_path[k] = cur;
+      if (s_out != nullptr) s_out[k - 1] = tk;
+    }
   }
+  if (lane == 0 && s_out != nullptr) s_out[n] = s_pred[cur];
   __syncwarp();
   return {n, 0};
 }
@@ -756,15 +764,18 @@ __device__ WalkOut tree_walk_warp(const int32_t *par_row, const int32_t *tok_row
 }
 
 // Writes accept_len, path, out_tokens and new_kv_len of sequence b (warp).
+// The emitted tokens come from s_out when the walk filled it, else from the
+// token and prediction rows in global memory.
 __device__ void write_walk(int b, int n, int L, const int32_t *tok_row, const int32_t *pred_row, const int32_t *s_path,
                            int max_path, int32_t *accept_len, int32_t *path, int32_t *out_tokens,
-                           int32_t *new_kv_len) {
+                           int32_t *new_kv_len, const int32_t *s_out = nullptr) {
   const int lane = threadIdx.x & 31;
   for (int k = lane; k < max_path; k += 32) {
     int pv = -1, ov = -1;
     if (n >= 0 && k <= n) {
       pv = s_path[k];
-      ov = (k < n) ? __ldg(tok_row + s_path[k + 1]) : __ldcg(pred_row + s_path[n]);
+      if (s_out != nullptr) ov = s_out[k];
+      else ov = (k < n) ? __ldg(tok_row + s_path[k + 1]) : __ldcg(pred_row + s_path[n]);
     }
     path[int64_t(b) * max_path + k] = pv;
     out_tokens[int64_t(b) * max_path + k] = ov;
@@ -795,15 +806,25 @@ __device__ __forceinline__ int64_t slot_off16(const KVParams &kv, int b, int s) 
   return (int64_t(pg) * 64 + (s & 63)) * kv.Hkv * kv.ch;
 }
 
+// The same from a cached page-table entry: pg = the entry of the slot's page.
+__device__ __forceinline__ int64_t slot_off16_pg(const KVParams &kv, int pg, int s) {
+  if (pg < 0 || pg >= kv.num_pages) return -1;
+  return (int64_t(pg) * 64 + (s & 63)) * kv.Hkv * kv.ch;
+}
+
 // Slot offsets of the moves of sequence b into s_src / s_dst (x = 1 .. n),
-// computed by one warp; returns false (and flags) on a bad page.
+// computed by one warp; returns false (and flags) on a bad page. With a paged
+// cache, s_pg (when given) holds the entries of pages L / 64 and L / 64 + 1,
+// which cover every slot a move touches (L .. L + T - 1, T <= 64).
 __device__ bool move_offsets(const KVParams &kv, int b, int L, int n, const int32_t *s_path, int64_t *s_src,
-                             int64_t *s_dst, int32_t *status) {
+                             int64_t *s_dst, int32_t *status, const int32_t *s_pg = nullptr) {
   const int lane = threadIdx.x & 31;
   int bad = 0;
+  const bool cached = s_pg != nullptr && kv.page_table != nullptr;
   for (int x = 1 + lane; x <= n; x += 32) {
-    const int64_t so = slot_off16(kv, b, L + s_path[x]);
-    const int64_t dst = slot_off16(kv, b, L + x);
+    const int ss = L + s_path[x], sd = L + x;
+    const int64_t so = cached ? slot_off16_pg(kv, s_pg[(ss >> 6) - (L >> 6)], ss) : slot_off16(kv, b, ss);
+    const int64_t dst = cached ? slot_off16_pg(kv, s_pg[(sd >> 6) - (L >> 6)], sd) : slot_off16(kv, b, sd);
     bad |= (so < 0 || dst < 0);
     s_src[x] = so;
     s_dst[x] = dst;
@@ -974,36 +995,46 @@ __global__ void __launch_bounds__(256) verify_sample_select_kernel(const StepPar
 // by programmatic dependent launch (it may start early and waits until launch
 // 1 has completed): the acceptance walk, its outputs, and the KV compaction.
 __global__ void __launch_bounds__(TAIL_THREADS) verify_tail_kernel(const StepParams p) {
-  __shared__ int32_t s_path[65];
+  __shared__ int32_t s_path[65], s_out[65], s_pg[2];
   __shared__ int64_t s_src[65], s_dst[65];
   __shared__ int s_n;
   const int b = blockIdx.x, Tm = p.tr.T_max;
   const int64_t rb = int64_t(b) * Tm;
   const int T = __ldg(p.tr.tree_len + b);
   const int L = __ldg(p.tr.kv_len + b);
-  // the tree's shape needs no prediction: computed while the argmax grid runs
+  // Everything that needs no prediction is done while the argmax grid runs:
+  // the tree's shape (with its tokens, which the walk then emits from
+  // registers) and, for a paged cache, the page-table entries of the tree's
+  // slots L .. L + T - 1 (two pages at most), which the compaction needs.
   const bool lens_ok = T >= 1 && T <= Tm && L >= 0 && L <= p.kv.capacity - T;
   TreeShape ts{};
-  if (threadIdx.x < 32 && lens_ok) ts = tree_shape_warp(p.tr.parent + rb, p.tr.tokens + rb, T);
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int e = -1;
+    if (lane < 2 && lens_ok && p.kv.page_table != nullptr && (L >> 6) + lane < p.kv.pages_per_seq)
+      e = __ldg(p.kv.page_table + int64_t(b) * p.kv.pages_per_seq + (L >> 6) + lane);
+    if (lens_ok) ts = tree_shape_warp(p.tr.parent + rb, p.tr.tokens + rb, T);
+    if (lane < 2) s_pg[lane] = e;
+  }
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (threadIdx.x < 32) {
     WalkOut w{-1, 0};
     if (T < 1 || T > Tm) w.bad = DREAMS_DATA_BAD_TREE_LEN;
     else if (L < 0 || L > p.kv.capacity - T) w.bad = DREAMS_DATA_BAD_KV_LEN;
     else if (ts.bad) w.bad = ts.bad;
-    else w = tree_walk_finish(ts, p.pred + rb, T, p.max_path, s_path);
+    else w = tree_walk_finish(ts, p.pred + rb, T, p.max_path, s_path, s_out);
     if (w.bad) {
       w.n = -1;
       if (threadIdx.x == 0) flag(p.status, w.bad);
     }
     write_walk(b, w.n, L, p.tr.tokens + rb, p.pred + rb, s_path, p.max_path, p.accept_len, p.path, p.out_tokens,
-               p.new_kv_len);
+               p.new_kv_len, s_out);
     if (p.pred_in_ws && T >= 1 && T <= Tm) {  // leave the workspace zero-filled
       __syncwarp();
       for (int x = threadIdx.x; x < T; x += 32) p.pred[rb + x] = 0;
     }
     bool ok = w.n > 0;
-    if (ok) ok = move_offsets(p.kv, b, L, w.n, s_path, s_src, s_dst, p.status);
+    if (ok) ok = move_offsets(p.kv, b, L, w.n, s_path, s_src, s_dst, p.status, s_pg);
     if (threadIdx.x == 0) s_n = ok ? w.n : 0;
   }
   __syncthreads();
