@@ -237,7 +237,12 @@ __global__ void __launch_bounds__(ORDER_THREADS) tree_attn_order_kernel(const At
   }
 }
 
-template <int D, bool ENT>
+// SPLIT: P is handed to the MMA thread in two halves, so that the first half
+// of PV_j runs while the softmax warps finish the tile (tree and
+// cross-attention rows, bound by the softmax-MMA chain), or whole (causal
+// rows, bound by the tensor pipe, where the extra wait between the PV halves
+// costs more than it saves). The host picks it by mode.
+template <int D, bool ENT, bool SPLIT>
 __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_constant__ TcParams P) {
   const AttnParams &p = P.a;
   constexpr int NR = D / 64;                     // 128-byte column regions of a row
@@ -251,7 +256,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ __align__(8) uint64_t bar_kf[NK], bar_ke[NK], bar_vf[NV], bar_ve[NV];
-  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_q, bar_drain, bar_never;
+  __shared__ __align__(8) uint64_t bar_s[2], bar_p[2], bar_ph[2], bar_q, bar_drain, bar_never;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_zero, s_flag, s_tma;
   __shared__ unsigned long long s_anc[64];
@@ -324,7 +329,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
   auto v_s = [&](int st) { return smem_base + Q_BYTES + uint32_t(NK + st) * KV_TILE; };
   const uint32_t kf0 = smem_u32(&bar_kf[0]), ke0 = smem_u32(&bar_ke[0]);
   const uint32_t vf0 = smem_u32(&bar_vf[0]), ve0 = smem_u32(&bar_ve[0]);
-  const uint32_t bs0 = smem_u32(&bar_s[0]), bp0 = smem_u32(&bar_p[0]);
+  const uint32_t bs0 = smem_u32(&bar_s[0]), bp0 = smem_u32(&bar_p[0]), bph0 = smem_u32(&bar_ph[0]);
   const uint32_t bq = smem_u32(&bar_q), bdrain = smem_u32(&bar_drain), bnever = smem_u32(&bar_never);
   const int t0 = rb * p.TB;  // first tree node of the row block
   const int c0 = split * p.chunk;
@@ -405,6 +410,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(bs0 + 8 * i, 1);
       tc::mbar_init(bp0 + 8 * i, 32 * n_act);
+      tc::mbar_init(bph0 + 8 * i, 32 * n_act);
     }
     tc::mbar_init(bdrain, 1);
     tc::mbar_init(bnever, 1);  // nothing arrives on it (the stall test hook waits on it)
@@ -610,12 +616,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
           tc::mma_ss(tmem + scol, ad, bd, IDESC_QK, k > 0 ? 1u : 0u);
         }
       };
-      // O_w += P_j V_j, w = j % 2
-      auto pv = [&](int j) {
+      // O_w += P_j V_j, w = j % 2, over the tile's first (h = 0) or last 64 keys
+      auto pv = [&](int j, int h) {
         const int w = j & 1, ii = j >> 1, vs = j % NV;
         const uint32_t scol = 256u * w, ocol = 256u * w + 128u;
 #pragma unroll
-        for (int ks = 0; ks < KT / 16; ++ks) {
+        for (int kk = 0; kk < KT / 32; ++kk) {
+          const int ks = h * (KT / 32) + kk;
           const uint64_t bd = vd0 + ((uint32_t(vs) * KV_TILE + ks * 2048) >> 4);
           tc::mma_ts(tmem + ocol, tmem + scol + ks * 8, bd, IDESC_PV, (ii > 0 || ks > 0) ? 1u : 0u);
         }
@@ -640,12 +647,21 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       // and V_j to the producer.
       for (int j = 0; j < ntiles && ok; ++j) {
         const int w = j & 1;
-        // P_j: the softmax warps arrive once one of them has also seen V_j
-        // and K_{j+2} land
+        // P_j over the first 64 keys (the softmax warps arrive once one of
+        // them has also seen V_j land): its PV half runs while they finish
+        // the tile; then the rest of P_j (K_{j+2} landed as well). Without
+        // SPLIT, P_j whole.
+        if constexpr (SPLIT) {
+          ok = tc::mbar_wait(bph0 + 8 * w, (j >> 1) & 1, abort_flag, wait_ns);
+          if (!ok) break;
+          tc::fence_after_sync();
+          pv(j, 0);
+        }
         ok = tc::mbar_wait(bp0 + 8 * w, (j >> 1) & 1, abort_flag, wait_ns);
         if (!ok) break;
         tc::fence_after_sync();
-        pv(j);
+        if constexpr (!SPLIT) pv(j, 0);
+        pv(j, 1);
         if (j + 2 < ntiles) {
           qk(j + 2);
           tc::mma_commit(bs0 + 8 * w);
@@ -730,80 +746,175 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         m_ref = mx;
         l *= corr;
       }
-      const float nmu = (m_ref == -INFINITY) ? 0.f : -m_ref;
-      // exponents scale * s - m two at a time (f32x2 FMA), their sum two at a
-      // time (f32x2 add), P as bf16 pairs
-      const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2), nmu2 = f32x2(nmu, nmu);
-      uint64_t acc2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
-      uint64_t wacc2 = f32x2(0.f, 0.f);  // entropy: sum of P e over the tile
+      if constexpr (SPLIT) {
+        // P in two halves of 64 keys: exponents scale * s - m two at a time
+        // (f32x2 FMA), their sum two at a time (f32x2 add), P as bf16 pairs
+        // over the first 64 columns of S, 32 keys per step
+        const float nmu = (m_ref == -INFINITY) ? 0.f : -m_ref;
+        const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2), nmu2 = f32x2(nmu, nmu);
+        uint64_t acc2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
+        uint64_t wacc2 = f32x2(0.f, 0.f);  // entropy: sum of P e over the tile
+        auto p_step = [&](int q4) {
+          uint32_t pk[16];
 #pragma unroll
-      for (int q4 = 0; q4 < KT / 32; ++q4) {
-        uint32_t pk[16];
+          for (int c = 0; c < 16; ++c) {
+            float e0, e1;
+            f32x2_split(ffma2(f32x2(__uint_as_float(sv[32 * q4 + 2 * c]), __uint_as_float(sv[32 * q4 + 2 * c + 1])),
+                              scale2, nmu2),
+                        e0, e1);
+            const float p0 = tc::ex2(e0), p1 = tc::ex2(e1);
+            acc2[c & 1] = fadd2(acc2[c & 1], f32x2(p0, p1));
+            // masked slots have e = -inf and P = 0: clamp e so that P e is 0, not NaN
+            if (ENT) wacc2 = ffma2(f32x2(p0, p1), f32x2(fmaxf(e0, -200.f), fmaxf(e1, -200.f)), wacc2);
+            pk[c] = pack_bf16x2(p0, p1);
+          }
+          tc::tmem_st16(tl + 16 * q4, pk);
+        };
+        p_step(0);
+        p_step(1);
+        // Before the first half goes to the MMA thread (with half the scores
+        // consumed, so that the registers allow it): slots past the sequence
+        // end may hold any bits (0 * NaN = NaN in the PV product), so their V
+        // rows are zeroed once the tile's copy has landed (a later landing
+        // would undo the zeros); and O follows a raised reference before
+        // PV_j's first half adds to it.
+        if (c1 - s0 < KT) {
+          const int st = j % NV;
+          if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag, wait_ns))) {
+            give_up();
+            ok = false;
+            break;
+          }
+          const int first = c1 - s0, nz = (KT - first) * NR * 8;
+          for (int i = 32 * (warp & 3) + lane; i < nz; i += 32 * n_act) {
+            const int r = first + i / (NR * 8), rc = i % (NR * 8);
+            const uint32_t dst = v_s(st) + (rc >> 3) * KV_REGION + r * 128 + ((rc & 7) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%1,%1,%1};" ::"r"(dst), "r"(0u) : "memory");
+          }
+          tc::fence_proxy_async_smem();
+        }
+        if (ii > 0 && __any_sync(0xffffffffu, resc)) {
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          float e0, e1;
-          f32x2_split(ffma2(f32x2(__uint_as_float(sv[32 * q4 + 2 * c]), __uint_as_float(sv[32 * q4 + 2 * c + 1])),
-                            scale2, nmu2),
-                      e0, e1);
-          const float p0 = tc::ex2(e0), p1 = tc::ex2(e1);
-          acc2[c & 1] = fadd2(acc2[c & 1], f32x2(p0, p1));
-          // masked slots have e = -inf and P = 0: clamp e so that P e is 0, not NaN
-          if (ENT) wacc2 = ffma2(f32x2(p0, p1), f32x2(fmaxf(e0, -200.f), fmaxf(e1, -200.f)), wacc2);
-          pk[c] = pack_bf16x2(p0, p1);
+          for (int c4 = 0; c4 < D / 32; ++c4) {
+            uint32_t ov[32];
+            tc::tmem_ld32(tl + 128 + c4 * 32, ov);
+            tc::tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
+            tc::tmem_st32(tl + 128 + c4 * 32, ov);
+          }
         }
-        tc::tmem_st16(tl + 16 * q4, pk);  // P (bf16 pairs) over the first 64 columns of S
-      }
-      {
-        float a0, a1, b0, b1;
-        f32x2_split(acc2[0], a0, a1);
-        f32x2_split(acc2[1], b0, b1);
-        l += (a0 + a1) + (b0 + b1);
-        if (ENT) {
-          f32x2_split(wacc2, a0, a1);
-          wsum += a0 + a1;
-        }
-      }
-      if (c1 - s0 < KT) {
-        // slots past the sequence end may hold any bits (0 * NaN = NaN in the
-        // PV product): zero those V rows before the MMA reads them, once the
-        // tile's copy has landed (a later landing would undo the zeros)
-        const int st = j % NV;
-        if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag, wait_ns))) {
+        // One thread also waits for the copies the MMA thread needs next, V_j
+        // for the first half of PV_j, then K_{j+2} for QK_{j+2} (usually
+        // landed by now; the waits overlap the TMEM stores): the MMA thread
+        // then waits for P alone.
+        bool kv_ok = true;
+        if (warp == 4 * wg && lane == 0)
+          kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag, wait_ns);
+        if (!__all_sync(0xffffffffu, kv_ok)) {
           give_up();
           ok = false;
           break;
         }
-        const int first = c1 - s0, nz = (KT - first) * NR * 8;
-        for (int i = 32 * (warp & 3) + lane; i < nz; i += 32 * n_act) {
-          const int r = first + i / (NR * 8), rc = i % (NR * 8);
-          const uint32_t dst = v_s(st) + (rc >> 3) * KV_REGION + r * 128 + ((rc & 7) << 4);
-          asm volatile("st.shared.v4.b32 [%0], {%1,%1,%1,%1};" ::"r"(dst), "r"(0u) : "memory");
+        tc::tmem_wait_st();
+        tc::fence_before_sync();
+        tc::mbar_arrive(bph0 + 8 * wg);
+        p_step(2);
+        p_step(3);
+        {
+          float a0, a1, b0, b1;
+          f32x2_split(acc2[0], a0, a1);
+          f32x2_split(acc2[1], b0, b1);
+          l += (a0 + a1) + (b0 + b1);
+          if (ENT) {
+            f32x2_split(wacc2, a0, a1);
+            wsum += a0 + a1;
+          }
         }
-        tc::fence_proxy_async_smem();
-      }
-      if (ii > 0 && __any_sync(0xffffffffu, resc)) {
-#pragma unroll
-        for (int c4 = 0; c4 < D / 32; ++c4) {
-          uint32_t ov[32];
-          tc::tmem_ld32(tl + 128 + c4 * 32, ov);
-          tc::tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
-          tc::tmem_st32(tl + 128 + c4 * 32, ov);
+        if (warp == 4 * wg && lane == 0)
+          kv_ok = j + 2 >= ntiles ||
+                  tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag, wait_ns);
+        if (!__all_sync(0xffffffffu, kv_ok)) {
+          give_up();
+          ok = false;
+          break;
         }
-      }
-      // One thread also waits for the copies the MMA thread needs next, V_j
-      // and K_{j+2} (usually landed by now; the wait overlaps the TMEM
-      // stores): the MMA thread then waits for P_j alone.
-      bool kv_ok = true;
-      if (warp == 4 * wg && lane == 0)
-        kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag, wait_ns) &&
-                (j + 2 >= ntiles ||
-                 tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag, wait_ns));
-      if (!__all_sync(0xffffffffu, kv_ok)) {
-        give_up();
-        ok = false;
-        break;
+      } else {
+        const float nmu = (m_ref == -INFINITY) ? 0.f : -m_ref;
+        // exponents scale * s - m two at a time (f32x2 FMA), their sum two at a
+        // time (f32x2 add), P as bf16 pairs
+        const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2), nmu2 = f32x2(nmu, nmu);
+        uint64_t acc2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
+        uint64_t wacc2 = f32x2(0.f, 0.f);  // entropy: sum of P e over the tile
+#pragma unroll
+        for (int q4 = 0; q4 < KT / 32; ++q4) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            float e0, e1;
+            f32x2_split(ffma2(f32x2(__uint_as_float(sv[32 * q4 + 2 * c]), __uint_as_float(sv[32 * q4 + 2 * c + 1])),
+                              scale2, nmu2),
+                        e0, e1);
+            const float p0 = tc::ex2(e0), p1 = tc::ex2(e1);
+            acc2[c & 1] = fadd2(acc2[c & 1], f32x2(p0, p1));
+            // masked slots have e = -inf and P = 0: clamp e so that P e is 0, not NaN
+            if (ENT) wacc2 = ffma2(f32x2(p0, p1), f32x2(fmaxf(e0, -200.f), fmaxf(e1, -200.f)), wacc2);
+            pk[c] = pack_bf16x2(p0, p1);
+          }
+          tc::tmem_st16(tl + 16 * q4, pk);  // P (bf16 pairs) over the first 64 columns of S
+        }
+        {
+          float a0, a1, b0, b1;
+          f32x2_split(acc2[0], a0, a1);
+          f32x2_split(acc2[1], b0, b1);
+          l += (a0 + a1) + (b0 + b1);
+          if (ENT) {
+            f32x2_split(wacc2, a0, a1);
+            wsum += a0 + a1;
+          }
+        }
+        if (c1 - s0 < KT) {
+          // slots past the sequence end may hold any bits (0 * NaN = NaN in the
+          // PV product): zero those V rows before the MMA reads them, once the
+          // tile's copy has landed (a later landing would undo the zeros)
+          const int st = j % NV;
+          if (!__all_sync(0xffffffffu, tc::mbar_wait(vf0 + 8 * st, (j / NV) & 1, abort_flag, wait_ns))) {
+            give_up();
+            ok = false;
+            break;
+          }
+          const int first = c1 - s0, nz = (KT - first) * NR * 8;
+          for (int i = 32 * (warp & 3) + lane; i < nz; i += 32 * n_act) {
+            const int r = first + i / (NR * 8), rc = i % (NR * 8);
+            const uint32_t dst = v_s(st) + (rc >> 3) * KV_REGION + r * 128 + ((rc & 7) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%1,%1,%1};" ::"r"(dst), "r"(0u) : "memory");
+          }
+          tc::fence_proxy_async_smem();
+        }
+        if (ii > 0 && __any_sync(0xffffffffu, resc)) {
+#pragma unroll
+          for (int c4 = 0; c4 < D / 32; ++c4) {
+            uint32_t ov[32];
+            tc::tmem_ld32(tl + 128 + c4 * 32, ov);
+            tc::tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
+            tc::tmem_st32(tl + 128 + c4 * 32, ov);
+          }
+        }
+        // One thread also waits for the copies the MMA thread needs next, V_j
+        // and K_{j+2} (usually landed by now; the wait overlaps the TMEM
+        // stores): the MMA thread then waits for P_j alone.
+        bool kv_ok = true;
+        if (warp == 4 * wg && lane == 0)
+          kv_ok = tc::mbar_wait(vf0 + 8 * (j % NV), (j / NV) & 1, abort_flag, wait_ns) &&
+                  (j + 2 >= ntiles ||
+                   tc::mbar_wait(kf0 + 8 * ((j + 2) % NK), ((j + 2) / NK) & 1, abort_flag, wait_ns));
+        if (!__all_sync(0xffffffffu, kv_ok)) {
+          give_up();
+          ok = false;
+          break;
+        }
       }
       tc::tmem_wait_st();
       tc::fence_before_sync();
@@ -1166,9 +1277,10 @@ template <int D, bool ENT>
 dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_cache_t *kv, const void *k,
                        const void *v, int B, int64_t q_stride_b, int64_t q_stride_t, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<D>();
+  const void *kernel = a.mode == ATTN_CAUSAL ? reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, false>)
+                                              : reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, true>);
   {
-    const dreams_status_t st =
-        ensure_max_dynamic_smem(reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT>), int(smem));
+    const dreams_status_t st = ensure_max_dynamic_smem(kernel, int(smem));
     if (st != DREAMS_OK) return st;
   }
   TcParams P;
@@ -1187,8 +1299,7 @@ dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_
   }
   const int64_t ctas = int64_t(B) * pl.nsplit * a.Hkv * pl.nrb;
   void *args_attn[] = {&P};
-  cudaError_t e = launch_pdl(reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT>), dim3(unsigned(ctas)),
-                             dim3(THREADS), smem, stream, pl.ordered, args_attn);
+  cudaError_t e = launch_pdl(kernel, dim3(unsigned(ctas)), dim3(THREADS), smem, stream, pl.ordered, args_attn);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return DREAMS_ERR_CUDA;
