@@ -241,9 +241,13 @@ __global__ void __launch_bounds__(ORDER_THREADS) tree_attn_order_kernel(const At
 // of PV_j runs while the softmax warps finish the tile (tree and
 // cross-attention rows, bound by the softmax-MMA chain), or whole (causal
 // rows, bound by the tensor pipe, where the extra wait between the PV halves
-// costs more than it saves). The host picks it by mode.
-template <int D, bool ENT, bool SPLIT>
+// costs more than it saves). VREL (with SPLIT): a V stage goes back to the
+// producer as soon as its PV has completed (one more commit per tile) rather
+// than at the next wake-up of the softmax warps: worth it where the copies
+// land late, on paged caches. The host picks both by mode and cache layout.
+template <int D, bool ENT, bool SPLIT, bool VREL>
 __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_constant__ TcParams P) {
+  static_assert(SPLIT || !VREL, "the early V release goes with the two-half hand-off");
   const AttnParams &p = P.a;
   constexpr int NR = D / 64;                     // 128-byte column regions of a row
   constexpr uint32_t Q_REGION = ROWS * 128;      // 16 KB
@@ -662,6 +666,9 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         tc::fence_after_sync();
         if constexpr (!SPLIT) pv(j, 0);
         pv(j, 1);
+        // with VREL, V_j's stage goes back to the producer as soon as PV_j
+        // has completed, ahead of QK_{j+2} (an arrival on its empty barrier)
+        if constexpr (VREL) tc::mma_commit(ve0 + 8 * (j % NV));
         if (j + 2 < ntiles) {
           qk(j + 2);
           tc::mma_commit(bs0 + 8 * w);
@@ -688,12 +695,13 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
         break;
       }
       // S_j is complete, and so (issued earlier) is this warpgroup's previous
-      // PV, so O may be rescaled below. The K stage of tile j and the V stage
-      // of tile j - 2 (read by that PV) go back to the producer.
+      // PV, so O may be rescaled below. The K stage of tile j and (unless the
+      // MMA thread's commit already did, VREL) the V stage of tile j - 2, read
+      // by that PV, go back to the producer.
       tc::fence_after_sync();
       if (warp == 4 * wg && lane == 0) {
         tc::mbar_arrive(ke0 + 8 * (j % NK));
-        if (j >= 2) tc::mbar_arrive(ve0 + 8 * ((j - 2) % NV));
+        if (!VREL && j >= 2) tc::mbar_arrive(ve0 + 8 * ((j - 2) % NV));  // (with VREL: the MMA thread's commit)
       }
       uint32_t sv[KT];
 #pragma unroll
@@ -1277,8 +1285,11 @@ template <int D, bool ENT>
 dreams_status_t launch(const AttnParams &a, const AttnPlan &pl, const dreams_kv_cache_t *kv, const void *k,
                        const void *v, int B, int64_t q_stride_b, int64_t q_stride_t, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<D>();
-  const void *kernel = a.mode == ATTN_CAUSAL ? reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, false>)
-                                              : reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, true>);
+  const void *kernel =
+      a.mode == ATTN_CAUSAL
+          ? reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, false, false>)
+          : (kv->page_table != nullptr ? reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, true, true>)
+                                       : reinterpret_cast<const void *>(tree_attn_tc_kernel<D, ENT, true, false>));
   {
     const dreams_status_t st = ensure_max_dynamic_smem(kernel, int(smem));
     if (st != DREAMS_OK) return st;
