@@ -122,18 +122,27 @@ def attn_flops(w: W.Workload) -> int:
                    for b in range(w.B)))
 
 
+def code_sha256(path: str) -> str:
+    """sha256 of a C++/CUDA source with its comments and blank lines removed:
+    it changes with the code, not with a comment edit."""
+    import hashlib
+    import re
+    text = open(path).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    lines = [re.sub(r"//.*$", "", line).rstrip() for line in text.splitlines()]
+    return hashlib.sha256("\n".join(line for line in lines if line).encode()).hexdigest()
+
+
 def measured_traffic(kernel: str, workload: str):
     """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
-    kernel source has not changed since it was captured (else None)."""
-    import hashlib
+    kernel's code has not changed since it was captured (else None)."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             rec = json.load(f)[kernel]
-        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
-            sha = hashlib.sha256(f.read()).hexdigest()
+        sha = code_sha256(os.path.join(ROOT, rec["source"]))
     except (OSError, KeyError, ValueError):
         return None
-    if sha != rec["source_sha256"] or rec["workload"] != workload:
+    if sha != rec["code_sha256"] or rec["workload"] != workload:
         return None
     return int(rec["dram_bytes_per_launch"])
 

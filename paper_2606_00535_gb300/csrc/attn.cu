@@ -607,7 +607,8 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       const uint64_t vd0 = tc::smem_desc_sw128(v_s(0), KV_REGION, 1024);
       // The tensor pipe queues only about one MMA, so any latency in the
       // issuing thread between MMAs idles it: per tile the thread takes one
-      // wait, then issues PV_j and QK_{j+2} (16 MMAs) under one commit.
+      // wait, then issues PV_j and QK_{j+2} (16 MMAs) under one commit (with
+      // SPLIT, one wait before each half of PV_j).
       // S_j = Q K_j^T into warpgroup (j % 2)'s S buffer
       auto qk = [&](int j) {
         const int ks = j % NK;
@@ -648,7 +649,7 @@ __global__ void __launch_bounds__(THREADS, 1) tree_attn_tc_kernel(const __grid_c
       }
       // The commit after QK_{j+2} also covers PV_j (the pipe completes in
       // order): the softmax warps, woken by it, release the stages of K_{j+2}
-      // and V_j to the producer.
+      // and (without VREL) V_j to the producer.
       for (int j = 0; j < ntiles && ok; ++j) {
         const int w = j & 1;
         // P_j over the first 64 keys (the softmax warps arrive once one of
