@@ -34,6 +34,11 @@
 //                       queues about one MMA, so the thread must not stall
 //                       between MMAs: per tile it waits once (for P_j), then
 //                       issues PV_j and QK_{j+2} (16 MMAs) under one commit.
+//                       Tree and cross-attention rows hand P_j over in two
+//                       halves of 64 keys, so the first half of PV_j runs
+//                       while the softmax finishes the tile; on a paged cache
+//                       the thread also commits V_j's stage free right after
+//                       PV_j.
 //   warps 0-3, 4-7      two softmax warpgroups, one query row per thread. A
 //                       warpgroup owns one S/P buffer and its own O in TMEM
 //                       (256 columns each), so the two alternate over the
@@ -44,15 +49,17 @@
 //                       exceeds it by 2^8 (and only then rescales its O), and
 //                       writes P as bf16 over S. Woken by the commit after
 //                       QK_j (which also covers PV_{j-2}), one thread
-//                       releases the K stage of tile j and the V stage of
-//                       tile j - 2 to the producer; before the warpgroup
-//                       signals P_j it waits for V_j and K_{j+2} to land, so
-//                       that the MMA thread needs no other wait. Warps whose
-//                       rows are all padding sit out.
-// At the end the two warpgroups combine their (m, l, O) by log-sum-exp and
-// each thread writes its row's half of the columns with 16-byte stores: the
-// output, or the split partials that a merge kernel (chained by programmatic
-// dependent launch) combines. Every mbarrier wait is bounded (2 s); on a
+//                       releases the K stage of tile j and (unless the MMA
+//                       thread did) the V stage of tile j - 2 to the
+//                       producer; before the warpgroup signals P_j (or its
+//                       first half) it waits for V_j and K_{j+2} (or V_j) to
+//                       land, so that the MMA thread needs no other wait.
+//                       Warps whose rows are all padding sit out.
+// At the end the two warpgroups combine their (m, l, O) by log-sum-exp. A
+// block whose rows all lie inside the tensor leaves through TMA stores of the
+// output staged in shared memory; other blocks write each row's half of the
+// columns with 16-byte stores: the output, or the split partials that a merge
+// kernel (chained by programmatic dependent launch) combines. Every mbarrier wait is bounded (2 s); on a
 // timeout the CTA flags DREAMS_DATA_TIMEOUT, drains its copies and MMAs, frees
 // its TMEM and exits. The workspace holds no state between calls.
 #include <cuda.h>
