@@ -175,6 +175,35 @@ def _need_out(out: torch.Tensor, name: str, dtype, dev, numel: int) -> torch.Ten
     return out
 
 
+def _ws(workspace: Optional[torch.Tensor], dev):
+    """Pointer and byte size of a caller's workspace (contiguous, on dev), or
+    (None, 0)."""
+    if workspace is None:
+        return None, 0
+    if not isinstance(workspace, torch.Tensor) or workspace.device != dev or not workspace.is_contiguous():
+        raise ValueError(f"workspace must be a contiguous tensor on {dev}")
+    return _ptr(workspace), workspace.numel() * workspace.element_size()
+
+
+def _status(status: Optional[torch.Tensor], dev):
+    """Pointer to the caller's device status word (int32, on dev), or None."""
+    return None if status is None else _ptr(_need_out(status, "status", torch.int32, dev, 1))
+
+
+def _outputs(outputs: Optional[tuple], B: int, max_path: int, dev) -> tuple:
+    """(accept_len [B], path [B, max_path], out_tokens [B, max_path],
+    new_kv_len [B]): the caller's, checked, or new."""
+    if outputs is None:
+        return _walk_outputs(B, max_path, dev)
+    if len(outputs) != 4:
+        raise ValueError("outputs must be (accept_len, path, out_tokens, new_kv_len)")
+    acc, path, toks, nkl = outputs
+    return (_need_out(acc, "accept_len", torch.int32, dev, B),
+            _need_out(path, "path", torch.int32, dev, B * max_path),
+            _need_out(toks, "out_tokens", torch.int32, dev, B * max_path),
+            _need_out(nkl, "new_kv_len", torch.int32, dev, B))
+
+
 def _need(t: torch.Tensor, name: str, dtype, dev) -> torch.Tensor:
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
@@ -276,8 +305,8 @@ def tree_verify_attn_launches(kv: KVCache, tree: Tree, Hq: int) -> int:
     return int(_lib().dreams_tree_verify_attn_launches(ctypes.byref(kv._c), ctypes.byref(tree._c), Hq))
 
 
-VERIFY_STEP_LAUNCHES = 2
-VERIFY_STEP_SAMPLED_LAUNCHES = 3  # draw statistics, draw selection, walk + compaction  # dreams_verify_step: the argmax, then the walk and compaction
+VERIFY_STEP_LAUNCHES = 2  # dreams_verify_step: the argmax, then the walk and compaction
+VERIFY_STEP_SAMPLED_LAUNCHES = 3  # draw statistics, draw selection, walk + compaction
 
 
 def _q_strides(q: torch.Tensor) -> Tuple[int, int]:
@@ -317,8 +346,8 @@ def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, lay
         workspace = _workspace("attn", need, dev, stream)
     _call("dreams_tree_verify_attn", dev,
           _ptr(q), sb, stt, ctypes.byref(kv._c), layer, ctypes.byref(tree._c), Hq, float(scale), _ptr(out),
-          _ptr(lse), _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
-          _ptr(status), _stream(stream, dev))
+          _ptr(lse), *_ws(workspace, dev),
+          _status(status, dev), _stream(stream, dev))
     return out, lse
 
 
@@ -336,7 +365,7 @@ def vocab_argmax(logits: torch.Tensor, out: Optional[torch.Tensor] = None,
         workspace = _workspace("argmax", need, dev, stream)
     _call("dreams_vocab_argmax", dev,
           _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), _ptr(out),
-          _ptr(workspace), 0 if workspace is None else workspace.numel(), _stream(stream, dev))
+          *_ws(workspace, dev), _stream(stream, dev))
     return out
 
 
@@ -378,7 +407,7 @@ def vocab_sample(logits: torch.Tensor, temperature: float, uniforms: torch.Tenso
         workspace = _workspace("sample", need, dev, stream)
     _call("dreams_vocab_sample", dev,
           _ptr(x), F32 if x.dtype == torch.float32 else BF16, rows, V, int(x.stride(0)), float(temperature),
-          _ptr(uniforms), _ptr(out), _ptr(workspace), 0 if workspace is None else workspace.numel(),
+          _ptr(uniforms), _ptr(out), *_ws(workspace, dev),
           _stream(stream, dev))
     return out
 
@@ -411,8 +440,8 @@ def attention(q: torch.Tensor, kv: KVCache, q_len: torch.Tensor, kv_len: torch.T
     if workspace is None:
         workspace = _workspace("attention", need, dev, stream)
     _call("dreams_attention", dev, _ptr(q), sb, stt, ctypes.byref(kv._c), layer, _ptr(q_len), _ptr(kv_len), B,
-          T_max, Hq, float(scale), mode, _ptr(out), _ptr(lse), _ptr(ent), _ptr(workspace),
-          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
+          T_max, Hq, float(scale), mode, _ptr(out), _ptr(lse), _ptr(ent), *_ws(workspace, dev),
+          _status(status, dev), _stream(stream, dev))
     return out, lse, ent
 
 
@@ -442,8 +471,8 @@ def lm_head_argmax(hidden: torch.Tensor, weight: torch.Tensor, out: Optional[tor
     if workspace is None:
         workspace = _workspace("lm_head", need, dev, stream)
     _call("dreams_lm_head_argmax", dev, _ptr(hidden), rows, K, int(hidden.stride(0)), _ptr(weight), V,
-          int(weight.stride(0)), _ptr(out), _ptr(out_max), _ptr(workspace),
-          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
+          int(weight.stride(0)), _ptr(out), _ptr(out_max), *_ws(workspace, dev), _status(status, dev),
+          _stream(stream, dev))
     return (out, out_max) if want_max or out_max is not None else out
 
 
@@ -463,7 +492,7 @@ def visual_importance(attn: torch.Tensor, v0: int, n_vis: int, r: int, workspace
     if workspace is None:
         workspace = _workspace("importance", need, dev, stream)
     _call("dreams_visual_importance", dev, _ptr(attn), F32 if attn.dtype == torch.float32 else BF16, B, H, Q, K, v0,
-          n_vis, r, _ptr(imp), _ptr(keep), _ptr(workspace), 0 if workspace is None else workspace.numel(),
+          n_vis, r, _ptr(imp), _ptr(keep), *_ws(workspace, dev),
           _stream(stream, dev))
     return imp, keep
 
@@ -482,7 +511,7 @@ def accept_path(argmax: torch.Tensor, tree: Tree, max_path: int, status: Optiona
     _need(argmax, "argmax", torch.int32, dev)
     acc, path, toks, nkl = _walk_outputs(tree.B, max_path, dev)
     _call("dreams_accept_path", dev, _ptr(argmax), ctypes.byref(tree._c), max_path, _ptr(acc), _ptr(path),
-          _ptr(toks), _ptr(nkl), _ptr(status), _stream(stream, dev))
+          _ptr(toks), _ptr(nkl), _status(status, dev), _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
 
@@ -494,7 +523,7 @@ def kv_compact(kv: KVCache, kv_len: torch.Tensor, accept_len: torch.Tensor, path
         _need(t, n, torch.int32, dev)
     B, max_path = (int(x) for x in path.shape)
     _call("dreams_kv_compact", dev, ctypes.byref(kv._c), B, _ptr(kv_len), _ptr(accept_len), _ptr(path), max_path,
-          _ptr(status), _stream(stream, dev))
+          _status(status, dev), _stream(stream, dev))
 
 
 def verify_step_sampled_workspace_size(tree: Tree, V: int) -> int:
@@ -519,15 +548,16 @@ def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
         raise ValueError("logits must be [B, T_max, V] with uniformly strided contiguous rows")
     V = int(logits.shape[2])
     if argmax_out is not None:
-        _need(argmax_out, "argmax_out", torch.int32, dev)
-    acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
+        _need_out(argmax_out, "argmax_out", torch.int32, dev, tree.B * tree.T_max)
+    acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
+    st = _status(status, dev)
     need = verify_step_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step", need, dev, stream)
     _call("dreams_verify_step", dev,
           _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
           ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, _ptr(argmax_out), _ptr(acc), _ptr(path),
-          _ptr(toks), _ptr(nkl), _ptr(workspace), 0 if workspace is None else workspace.numel(), _ptr(status),
+          _ptr(toks), _ptr(nkl), *_ws(workspace, dev), st,
           _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
@@ -550,16 +580,17 @@ def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path:
         raise ValueError("uniforms must be [B, T_max]")
     V = int(logits.shape[2])
     if sample_out is not None:
-        _need(sample_out, "sample_out", torch.int32, dev)
-    acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
+        _need_out(sample_out, "sample_out", torch.int32, dev, tree.B * tree.T_max)
+    acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
+    st = _status(status, dev)
     need = verify_step_sampled_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step_sampled", need, dev, stream)
     _call("dreams_verify_step_sampled", dev,
           _ptr(logits), F32 if logits.dtype == torch.float32 else BF16, V, int(logits.stride(1)),
           ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature), _ptr(uniforms),
-          _ptr(sample_out), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(workspace),
-          0 if workspace is None else workspace.numel(), _ptr(status), _stream(stream, dev))
+          _ptr(sample_out), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), *_ws(workspace, dev),
+          st, _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 
 
@@ -588,11 +619,12 @@ def verify_step_speculative(target_logits: torch.Tensor, draft_logits: torch.Ten
         if tuple(t.shape) != (tree.B, tree.T_max):
             raise ValueError(f"{n} must be [B, T_max]")
     V = int(target_logits.shape[2])
-    acc, path, toks, nkl = outputs if outputs is not None else _walk_outputs(tree.B, max_path, dev)
+    acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
+    st = _status(status, dev)
     _call("dreams_verify_step_speculative", dev,
           _ptr(target_logits), _ptr(draft_logits), F32 if target_logits.dtype == torch.float32 else BF16, V,
           int(target_logits.stride(1)), ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature),
-          _ptr(u_accept), _ptr(u_resample), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), _ptr(status),
+          _ptr(u_accept), _ptr(u_resample), _ptr(acc), _ptr(path), _ptr(toks), _ptr(nkl), st,
           _stream(stream, dev))
     return {"accept_len": acc, "path": path, "out_tokens": toks, "new_kv_len": nkl}
 

@@ -244,3 +244,44 @@ def test_speculative_binding_checks_before_any_call():
         dreams.verify_step_speculative(tgt, tgt, tree, kv, 3, 1.0, torch.zeros((B, 2), dtype=torch.float32), u)
     with pytest.raises((TypeError, ValueError)):
         dreams.verify_step_speculative(tgt, tgt, tree, kv, 3, 1.0, u, u.double())
+
+
+def test_binding_checks_outputs_status_and_workspace():
+    """The verify-step wrappers check caller-provided outputs (dtype, and at
+    least the elements the kernels write), the status word (int32, one
+    element) and the workspace (a contiguous tensor on the tensors' device)
+    before any library call."""
+    B, T, V, P = 2, 4, 16, 3
+    tree = dreams.Tree(torch.full((B, T), -1, dtype=torch.int32), torch.zeros((B, T), dtype=torch.int32),
+                       torch.ones(B, dtype=torch.int32), torch.zeros(B, dtype=torch.int32))
+    k = torch.zeros((B, 8, 1, 64), dtype=torch.bfloat16)
+    kv = dreams.KVCache(k, k.clone())
+    lg = torch.zeros((B, T, V), dtype=torch.float32)
+    u = torch.zeros((B, T), dtype=torch.float32)
+    good = (torch.zeros(B, dtype=torch.int32), torch.zeros((B, P), dtype=torch.int32),
+            torch.zeros((B, P), dtype=torch.int32), torch.zeros(B, dtype=torch.int32))
+    short_path = (good[0], torch.zeros((B, P - 1), dtype=torch.int32), good[2], good[3])
+    wrong_dtype = (good[0].long(), good[1], good[2], good[3])
+    calls = [
+        lambda **kw: dreams.verify_step(lg, tree, kv, P, **kw),
+        lambda **kw: dreams.verify_step_sampled(lg, tree, kv, P, 1.0, u, **kw),
+        lambda **kw: dreams.verify_step_speculative(lg, lg, tree, kv, P, 1.0, u, u, **kw),
+    ]
+    for call in calls:
+        with pytest.raises(ValueError, match="path holds"):
+            call(outputs=short_path)
+        with pytest.raises(TypeError, match="accept_len must be"):
+            call(outputs=wrong_dtype)
+        with pytest.raises(ValueError, match="outputs must be"):
+            call(outputs=good[:3])
+        with pytest.raises(TypeError, match="status must be"):
+            call(outputs=good, status=torch.zeros(1, dtype=torch.int64))
+        with pytest.raises(ValueError, match="status holds"):
+            call(outputs=good, status=torch.zeros(0, dtype=torch.int32))
+    with pytest.raises(ValueError, match="argmax_out holds"):
+        dreams.verify_step(lg, tree, kv, P, argmax_out=torch.zeros(B * T - 1, dtype=torch.int32), outputs=good)
+    with pytest.raises(ValueError, match="sample_out holds"):
+        dreams.verify_step_sampled(lg, tree, kv, P, 1.0, u, sample_out=torch.zeros(B * T - 1, dtype=torch.int32),
+                                   outputs=good)
+    with pytest.raises(ValueError, match="workspace must be a contiguous tensor"):
+        dreams.verify_step(lg, tree, kv, P, outputs=good, workspace=torch.zeros((64, 4), dtype=torch.uint8).t())
