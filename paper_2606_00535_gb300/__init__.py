@@ -309,6 +309,15 @@ VERIFY_STEP_LAUNCHES = 2  # dreams_verify_step: the argmax, then the walk and co
 VERIFY_STEP_SAMPLED_LAUNCHES = 3  # draw statistics, draw selection, walk + compaction
 
 
+def _cache_covers(kv: "KVCache", B: int, D: Optional[int] = None) -> None:
+    """The cache holds (at least) the B sequences a call reads or writes, with
+    head dim D when given."""
+    if kv.B < B:
+        raise ValueError(f"the KV cache holds {kv.B} sequences, the call addresses {B}")
+    if D is not None and kv.D != D:
+        raise ValueError(f"q's head dim {D} differs from the cache's {kv.D}")
+
+
 def _q_strides(q: torch.Tensor) -> Tuple[int, int]:
     """(sequence stride, token stride) in elements of a bf16 [B, T, Hq, D]
     query tensor whose head rows are dense (a view into a fused QKV output
@@ -330,6 +339,9 @@ def tree_verify_attn(q: torch.Tensor, kv: KVCache, tree: Tree, scale: float, lay
     dev = q.device
     sb, stt = _q_strides(q)
     Hq = int(q.shape[2])
+    if tuple(q.shape[:2]) != (tree.B, tree.T_max):
+        raise ValueError(f"q must be [B, T_max, Hq, D] with the tree's B = {tree.B}, T_max = {tree.T_max}")
+    _cache_covers(kv, tree.B, int(q.shape[3]))
     if out is None:
         out = torch.empty(tuple(q.shape), dtype=torch.bfloat16, device=dev)
     _need(out, "out", torch.bfloat16, dev)
@@ -426,9 +438,12 @@ def attention(q: torch.Tensor, kv: KVCache, q_len: torch.Tensor, kv_len: torch.T
     lse, entropy); out is dense; lse and entropy are None unless asked."""
     dev = q.device
     sb, stt = _q_strides(q)
+    B, T_max, Hq = int(q.shape[0]), int(q.shape[1]), int(q.shape[2])
     for n, t in (("q_len", q_len), ("kv_len", kv_len)):
         _need(t, n, torch.int32, dev)
-    B, T_max, Hq = int(q.shape[0]), int(q.shape[1]), int(q.shape[2])
+        if t.numel() < B:
+            raise ValueError(f"{n} holds {t.numel()} entries, q has {B} sequences")
+    _cache_covers(kv, B, int(q.shape[3]))
     if out is None:
         out = torch.empty(tuple(q.shape), dtype=torch.bfloat16, device=dev)
     _need(out, "out", torch.bfloat16, dev)
@@ -521,7 +536,13 @@ def kv_compact(kv: KVCache, kv_len: torch.Tensor, accept_len: torch.Tensor, path
     dev = kv.k.device
     for n, t in (("kv_len", kv_len), ("accept_len", accept_len), ("path", path)):
         _need(t, n, torch.int32, dev)
+    if path.dim() != 2:
+        raise ValueError("path must be [B, max_path]")
     B, max_path = (int(x) for x in path.shape)
+    for n, t in (("kv_len", kv_len), ("accept_len", accept_len)):
+        if t.numel() < B:
+            raise ValueError(f"{n} holds {t.numel()} entries, path has {B} rows")
+    _cache_covers(kv, B)
     _call("dreams_kv_compact", dev, ctypes.byref(kv._c), B, _ptr(kv_len), _ptr(accept_len), _ptr(path), max_path,
           _status(status, dev), _stream(stream, dev))
 
@@ -551,6 +572,7 @@ def verify_step(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path: int,
         _need_out(argmax_out, "argmax_out", torch.int32, dev, tree.B * tree.T_max)
     acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
     st = _status(status, dev)
+    _cache_covers(kv, tree.B)
     need = verify_step_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step", need, dev, stream)
@@ -583,6 +605,7 @@ def verify_step_sampled(logits: torch.Tensor, tree: Tree, kv: KVCache, max_path:
         _need_out(sample_out, "sample_out", torch.int32, dev, tree.B * tree.T_max)
     acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
     st = _status(status, dev)
+    _cache_covers(kv, tree.B)
     need = verify_step_sampled_workspace_size(tree, V)
     if workspace is None:
         workspace = _workspace("step_sampled", need, dev, stream)
@@ -621,6 +644,7 @@ def verify_step_speculative(target_logits: torch.Tensor, draft_logits: torch.Ten
     V = int(target_logits.shape[2])
     acc, path, toks, nkl = _outputs(outputs, tree.B, max_path, dev)
     st = _status(status, dev)
+    _cache_covers(kv, tree.B)
     _call("dreams_verify_step_speculative", dev,
           _ptr(target_logits), _ptr(draft_logits), F32 if target_logits.dtype == torch.float32 else BF16, V,
           int(target_logits.stride(1)), ctypes.byref(tree._c), ctypes.byref(kv._c), max_path, float(temperature),

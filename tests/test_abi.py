@@ -285,3 +285,37 @@ def test_binding_checks_outputs_status_and_workspace():
                                    outputs=good)
     with pytest.raises(ValueError, match="workspace must be a contiguous tensor"):
         dreams.verify_step(lg, tree, kv, P, outputs=good, workspace=torch.zeros((64, 4), dtype=torch.uint8).t())
+
+
+def test_binding_checks_batch_and_head_dims():
+    """Queries that do not match the tree's (B, T_max), a head dim other than
+    the cache's, a cache with fewer sequences than the call addresses, and
+    length arrays shorter than the batch are refused before any call."""
+    B, T, H, D = 3, 4, 2, 64
+    tree = dreams.Tree(torch.full((B, T), -1, dtype=torch.int32), torch.zeros((B, T), dtype=torch.int32),
+                       torch.ones(B, dtype=torch.int32), torch.zeros(B, dtype=torch.int32))
+    k = torch.zeros((B, 16, H, D), dtype=torch.bfloat16)
+    kv = dreams.KVCache(k, k.clone())
+    small = dreams.KVCache(k[:2].contiguous(), k[:2].contiguous())
+    q = torch.zeros((B, T, H, D), dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="the tree's B"):
+        dreams.tree_verify_attn(q[:2], kv, tree, 0.1)
+    with pytest.raises(ValueError, match="the tree's B"):
+        dreams.tree_verify_attn(torch.zeros((B, T + 1, H, D), dtype=torch.bfloat16), kv, tree, 0.1)
+    with pytest.raises(ValueError, match="head dim"):
+        dreams.tree_verify_attn(torch.zeros((B, T, H, 2 * D), dtype=torch.bfloat16), kv, tree, 0.1)
+    with pytest.raises(ValueError, match="holds 2 sequences"):
+        dreams.tree_verify_attn(q, small, tree, 0.1)
+    lens = torch.ones(B, dtype=torch.int32)
+    with pytest.raises(ValueError, match="q_len holds 2 entries"):
+        dreams.attention(q, kv, lens[:2], lens, 0.1, dreams.ATTN_FULL)
+    with pytest.raises(ValueError, match="holds 2 sequences"):
+        dreams.attention(q, small, lens, lens, 0.1, dreams.ATTN_FULL)
+    lg = torch.zeros((B, T, 8), dtype=torch.float32)
+    with pytest.raises(ValueError, match="holds 2 sequences"):
+        dreams.verify_step(lg, tree, small, 3)
+    path = torch.zeros((B, 3), dtype=torch.int32)
+    with pytest.raises(ValueError, match="kv_len holds 2 entries"):
+        dreams.kv_compact(kv, lens[:2], lens, path)
+    with pytest.raises(ValueError, match="holds 2 sequences"):
+        dreams.kv_compact(small, lens, lens, path)
