@@ -171,7 +171,7 @@ def _rows_view(logits: torch.Tensor) -> torch.Tensor:
 def _need_out(out: torch.Tensor, name: str, dtype, dev, numel: int) -> torch.Tensor:
     _need(out, name, dtype, dev)
     if out.numel() < numel:
-        raise ValueError(f"{name} holds {out.numel()} elements, {numel} are written")
+        raise ValueError(f"{name} holds {out.numel()} elements, the call uses {numel}")
     return out
 
 
@@ -523,7 +523,7 @@ def accept_path(argmax: torch.Tensor, tree: Tree, max_path: int, status: Optiona
                 stream=None) -> dict:
     """Greedy acceptance over the trees. Returns a dict of device tensors."""
     dev = tree.parent.device
-    _need(argmax, "argmax", torch.int32, dev)
+    _need_out(argmax, "argmax", torch.int32, dev, tree.B * tree.T_max)
     acc, path, toks, nkl = _walk_outputs(tree.B, max_path, dev)
     _call("dreams_accept_path", dev, _ptr(argmax), ctypes.byref(tree._c), max_path, _ptr(acc), _ptr(path),
           _ptr(toks), _ptr(nkl), _status(status, dev), _stream(stream, dev))

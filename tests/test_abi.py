@@ -319,3 +319,5 @@ def test_binding_checks_batch_and_head_dims():
         dreams.kv_compact(kv, lens[:2], lens, path)
     with pytest.raises(ValueError, match="holds 2 sequences"):
         dreams.kv_compact(small, lens, lens, path)
+    with pytest.raises(ValueError, match="argmax holds"):
+        dreams.accept_path(torch.zeros(B * T - 1, dtype=torch.int32), tree, 3)
