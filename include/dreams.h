@@ -93,6 +93,11 @@ typedef enum dreams_dtype { DREAMS_F32 = 0, DREAMS_BF16 = 1 } dreams_dtype_t;
  *    capacity must equal pages_per_seq * page_size. Only page_size 64.
  *  - layer l's cache starts layer_stride elements after layer l-1's (k and v
  *    alike). k, v and layer_stride * 2 bytes must be 16-byte aligned.
+ *  - The struct carries no batch size: a call that addresses sequences
+ *    0 .. B-1 reads (and the compaction writes) their slots, so the caller's
+ *    buffers must hold at least B sequences (contiguous: B * capacity slots
+ *    per layer; paged: B rows of the page table). The Python binding checks
+ *    this; the library cannot.
  */
 typedef struct dreams_kv_cache {
   void *k;
