@@ -605,3 +605,50 @@ def test_verify_step_ragged_repeat(dreams, dtype, aligned):
         ko, vo, ost = oracle.kv_compact(ko, vo, lay, kl, ref["accept_len"], ref["path"])
         assert ost == 0
         assert np.array_equal(W.bits(kv.k.cpu()), ko) and np.array_equal(W.bits(kv.v.cpu()), vo)
+
+
+@pytest.mark.parametrize("tail", [1, 63, 64, 65, 127])
+def test_attention_paged_ragged_tails(dreams, tail):
+    """A paged cache (pages in a seeded random order) whose sequences end `tail`
+    keys into their last 128-key tile: before, at and after the 64-key halves
+    in which P goes to the MMA thread, for a long sequence split over several
+    CTAs, a medium one and a one-tile one. The paged run equals the contiguous
+    run bit for bit, and both match the oracle."""
+    rng = np.random.default_rng(1000 + tail)
+    B, Hq, Hkv, D, T, cap = 3, 8, 2, 128, 24, 1024
+    tl = np.array([24, 9, 1], np.int32)
+    tiles = np.array([7, 2, 0])
+    kl = (128 * tiles + tail - tl).astype(np.int32)
+    kl[2] = max(0, tail - 1)
+    assert (kl >= 0).all() and (kl + tl <= cap).all()
+    par = np.stack([W.random_tree(rng, T) for _ in range(B)]).astype(np.int32)
+    for b in range(B):
+        par[b, tl[b]:] = -1
+    q = W.bf16(rng.standard_normal((B, T, Hq, D), dtype=np.float32))
+    k = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    v = W.bf16(rng.standard_normal((B, cap, Hkv, D), dtype=np.float32))
+    pps = cap // 64
+    perm = torch.randperm(B * pps, generator=torch.Generator().manual_seed(tail))
+    table = perm.view(B, pps).to(torch.int32)
+    kp = torch.empty((B * pps, 64, Hkv, D), dtype=torch.bfloat16)
+    vp = torch.empty_like(kp)
+    for b in range(B):
+        for pg in range(pps):
+            kp[table[b, pg]] = k[b, 64 * pg:64 * (pg + 1)]
+            vp[table[b, pg]] = v[b, 64 * pg:64 * (pg + 1)]
+    tree = dreams.Tree(torch.from_numpy(par).cuda(), torch.zeros((B, T), dtype=torch.int32, device="cuda"),
+                       torch.from_numpy(tl).cuda(), torch.from_numpy(kl).cuda())
+    scale = 1.0 / np.sqrt(D)
+    st = _status()
+    res = []
+    for kv in (dreams.KVCache(k.cuda(), v.cuda()), dreams.KVCache(kp.cuda(), vp.cuda(), table.cuda())):
+        res.append(dreams.tree_verify_attn(q.cuda(), kv, tree, scale, want_lse=True, status=st))
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for b in range(B):
+        for x, y in zip(res[0], res[1]):
+            assert torch.equal(x[b, :tl[b]], y[b, :tl[b]])
+    ref, ref_lse, sel, ost = oracle.tree_attention(W.bits(q), W.bits(k), W.bits(v), oracle.KVLayout(cap, Hkv, D),
+                                                   par, tl, kl, Hq, scale)
+    assert ost == 0
+    compare_attention(res[1][0], res[1][1], ref, ref_lse, sel)
